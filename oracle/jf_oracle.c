@@ -1,0 +1,557 @@
+/*
+ * jf_oracle.c -- CPU oracle for the Jacobi-decoding hot path (TEST INFRASTRUCTURE ONLY).
+ *
+ * This file is the plain, slow reference that the CUDA path is checked against. Only the
+ * test suite, the package's smoke check and the benchmark's CPU-baseline leg may load it.
+ * It shares no code, header, table or constant generator with the CUDA path.
+ *
+ * What it computes (Jacobi Forcing, arXiv 2512.14681):
+ *   - the causal decoder-only transformer p_theta of Sec. 2.1 (Eq. 1), in the Qwen2.5 shape
+ *     named in Sec. 4.1: RMSNorm -> Q/K/V -> rotary embedding -> grouped-query causal
+ *     attention over the exact KV cache of the committed prefix -> O projection + residual
+ *     -> RMSNorm -> SwiGLU MLP + residual; final RMSNorm -> LM head;
+ *   - one forward over M in-flight rows with the block-causal ("tree") mask, which is how
+ *     Eq. 3 solves all n conditionals of a Jacobi block in one pass; multi-block decoding
+ *     and rejection recycling (Sec. 3.2, Algorithm 1) only add segments to this mask;
+ *   - the greedy prediction g = argmax(logits) of Algorithm 1 (verification step);
+ *   - the KV commit / cache trim of Algorithm 1 (keep only the accepted rows' K/V).
+ *
+ * Arithmetic: fp64 throughout. For a bf16 model the tensors a bf16 model stores or streams
+ * are held at bf16 precision: the weights, the K/V cache, and the activations that enter a
+ * matrix product (normalised hidden states, rotated queries, attention output, SwiGLU
+ * product). Each is rounded to the nearest bf16 value (ties to even) at that point and the
+ * arithmetic continues in fp64. The greedy argmax is decided on the logits rounded to fp32,
+ * the precision in which the CUDA path takes the same decision; ties go to the lowest id.
+ *
+ * Random weights use a counter-based generator written from its published definition:
+ * SplitMix64 (Steele, Lea & Flood, OOPSLA 2014; constants of Vigna's public-domain
+ * splitmix64.c) feeding the Box-Muller transform (Box & Muller, 1958).
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+#define ORC_OK 0
+#define ORC_EINVAL 1
+#define ORC_ENOMEM 2
+
+/* ------------------------------------------------------------------------------------------
+ * Counter-based random numbers.
+ * SplitMix64: state advances by gamma = 0x9E3779B97F4A7C15, output = mix(state).
+ * The i-th output (i = 0, 1, ...) of a stream started at state s is mix(s + (i + 1) * gamma).
+ * ---------------------------------------------------------------------------------------- */
+static uint64_t orc_mix64(uint64_t z) {
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ULL;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBULL;
+    return z ^ (z >> 31);
+}
+
+uint64_t orc_sm64(uint64_t state, uint64_t i) {
+    return orc_mix64(state + (i + 1ULL) * 0x9E3779B97F4A7C15ULL);
+}
+
+/* Standard normal deviate number e of the stream keyed by (seed, tid):
+ * stream state s = output tid of the stream seeded with `seed`; pair j = e / 2 draws
+ * a = output 2j, b = output 2j+1; u1 = (a>>11 + 1) 2^-53 in (0,1], u2 = (b>>11) 2^-53 in [0,1);
+ * z0 = sqrt(-2 ln u1) cos(2 pi u2) (even e), z1 = sqrt(-2 ln u1) sin(2 pi u2) (odd e). */
+double orc_normal(uint64_t seed, uint64_t tid, uint64_t e) {
+    const double two53 = 9007199254740992.0;
+    uint64_t s = orc_sm64(seed, tid);
+    uint64_t j = e >> 1;
+    uint64_t a = orc_sm64(s, 2 * j);
+    uint64_t b = orc_sm64(s, 2 * j + 1);
+    double u1 = ((double)(a >> 11) + 1.0) / two53;
+    double u2 = (double)(b >> 11) / two53;
+    double rad = sqrt(-2.0 * log(u1));
+    double ang = 2.0 * 3.14159265358979323846 * u2;
+    return (e & 1) ? rad * sin(ang) : rad * cos(ang);
+}
+
+/* Nearest bf16 value of x (ties to even), returned as a double. bf16 keeps 8 significant
+ * bits and fp32's exponent range; x * 2^(7-e) is exact, rint() rounds half to even. */
+double orc_round_bf16(double x) {
+    if (x == 0.0 || !isfinite(x)) return x;
+    int e;
+    frexp(x, &e);           /* x = f * 2^e with 0.5 <= |f| < 1 */
+    e -= 1;                 /* now 1 <= |x| * 2^-e < 2 */
+    if (e < -126) e = -126; /* subnormal range of bf16 */
+    double scaled = ldexp(x, 7 - e);
+    return ldexp(rint(scaled), e - 7);
+}
+
+/* bf16 bit pattern of a value that is already a bf16 value (used for storage only). */
+static uint16_t orc_bf16_bits(double v) {
+    float f = (float)v;
+    uint32_t u;
+    memcpy(&u, &f, 4);
+    return (uint16_t)(u >> 16);
+}
+
+static double orc_bf16_value(uint16_t b) {
+    uint32_t u = ((uint32_t)b) << 16;
+    float f;
+    memcpy(&f, &u, 4);
+    return (double)f;
+}
+
+/* ------------------------------------------------------------------------------------------
+ * Model.
+ * ---------------------------------------------------------------------------------------- */
+typedef struct {
+    int n_layers, d_model, n_heads, n_kv_heads, head_dim, d_ff, vocab;
+    double rms_eps, rope_theta;
+    int bf16; /* 1: bf16 model (see header), 0: fp32 model */
+} orc_config;
+
+/* Logical tensor ids: 0 embedding [V,d], 1 LM head [V,d], 2 final-norm gain [1,d];
+ * layer l at 8 + 16 l: +0 attention-norm gain [1,d], +1 Wq [Hq hd, d], +2 Wk [Hkv hd, d],
+ * +3 Wv [Hkv hd, d], +4 Wo [d, Hq hd], +5 MLP-norm gain [1,d], +6 W_gate [F,d],
+ * +7 W_up [F,d], +8 W_down [d,F]. Matrices are [out, in], row-major. */
+enum { T_EMBED = 0, T_LMHEAD = 1, T_FNORM = 2 };
+enum { L_ANORM = 0, L_WQ, L_WK, L_WV, L_WO, L_MNORM, L_WG, L_WU, L_WD, L_COUNT };
+#define ORC_LAYER_BASE 8
+#define ORC_LAYER_STRIDE 16
+
+typedef struct {
+    long rows, cols;
+    float* f32;     /* fp32 model storage */
+    uint16_t* b16;  /* bf16 model storage (matrices); gains are stored in f32 */
+} orc_tensor;
+
+typedef struct {
+    orc_config cfg;
+    int n_tensors;
+    orc_tensor* t;
+} orc_model;
+
+int orc_tensor_shape(const orc_config* c, int tid, long* rows, long* cols) {
+    long d = c->d_model, qd = (long)c->n_heads * c->head_dim, kvd = (long)c->n_kv_heads * c->head_dim;
+    if (tid == T_EMBED || tid == T_LMHEAD) { *rows = c->vocab; *cols = d; return ORC_OK; }
+    if (tid == T_FNORM) { *rows = 1; *cols = d; return ORC_OK; }
+    if (tid < ORC_LAYER_BASE) return ORC_EINVAL;
+    int l = (tid - ORC_LAYER_BASE) / ORC_LAYER_STRIDE, w = (tid - ORC_LAYER_BASE) % ORC_LAYER_STRIDE;
+    if (l >= c->n_layers || w >= L_COUNT) return ORC_EINVAL;
+    switch (w) {
+        case L_ANORM: case L_MNORM: *rows = 1; *cols = d; break;
+        case L_WQ: *rows = qd; *cols = d; break;
+        case L_WK: case L_WV: *rows = kvd; *cols = d; break;
+        case L_WO: *rows = d; *cols = qd; break;
+        case L_WG: case L_WU: *rows = c->d_ff; *cols = d; break;
+        case L_WD: *rows = d; *cols = c->d_ff; break;
+        default: return ORC_EINVAL;
+    }
+    return ORC_OK;
+}
+
+static int orc_is_gain(int tid) {
+    if (tid == T_FNORM) return 1;
+    if (tid < ORC_LAYER_BASE) return 0;
+    int w = (tid - ORC_LAYER_BASE) % ORC_LAYER_STRIDE;
+    return w == L_ANORM || w == L_MNORM;
+}
+
+static int orc_tid_valid(const orc_config* c, int tid) {
+    long r, k;
+    return orc_tensor_shape(c, tid, &r, &k) == ORC_OK;
+}
+
+static inline double orc_w(const orc_tensor* t, long idx) {
+    return t->b16 ? orc_bf16_value(t->b16[idx]) : (double)t->f32[idx];
+}
+
+static void orc_w_store(orc_tensor* t, long idx, double v, int bf16) {
+    if (t->b16) t->b16[idx] = orc_bf16_bits(orc_round_bf16(v));
+    else t->f32[idx] = bf16 ? (float)orc_round_bf16(v) : (float)v;
+}
+
+void orc_model_free(orc_model* m) {
+    if (!m) return;
+    for (int i = 0; i < m->n_tensors; i++) { free(m->t[i].f32); free(m->t[i].b16); }
+    free(m->t);
+    free(m);
+}
+
+orc_model* orc_model_create(const orc_config* c) {
+    if (c->n_layers < 1 || c->d_model < 1 || c->n_heads < 1 || c->n_kv_heads < 1 ||
+        c->head_dim < 2 || (c->head_dim & 1) || c->n_heads % c->n_kv_heads || c->d_ff < 1 ||
+        c->vocab < 2)
+        return NULL;
+    orc_model* m = (orc_model*)calloc(1, sizeof(orc_model));
+    if (!m) return NULL;
+    m->cfg = *c;
+    m->n_tensors = ORC_LAYER_BASE + ORC_LAYER_STRIDE * c->n_layers;
+    m->t = (orc_tensor*)calloc((size_t)m->n_tensors, sizeof(orc_tensor));
+    if (!m->t) { free(m); return NULL; }
+    for (int tid = 0; tid < m->n_tensors; tid++) {
+        long r, k;
+        if (orc_tensor_shape(c, tid, &r, &k) != ORC_OK) continue;
+        orc_tensor* t = &m->t[tid];
+        t->rows = r; t->cols = k;
+        if (c->bf16 && !orc_is_gain(tid)) t->b16 = (uint16_t*)calloc((size_t)(r * k), 2);
+        else t->f32 = (float*)calloc((size_t)(r * k), 4);
+        if (!t->b16 && !t->f32) { orc_model_free(m); return NULL; }
+        if (orc_is_gain(tid)) for (long i = 0; i < r * k; i++) t->f32[i] = 1.0f;
+    }
+    return m;
+}
+
+/* Every matrix entry = std * N(0,1) deviate (orc_normal with the tensor id as stream key),
+ * rounded to the model's storage precision; RMSNorm gains stay 1.0. */
+void orc_init_random(orc_model* m, uint64_t seed, double std) {
+    for (int tid = 0; tid < m->n_tensors; tid++) {
+        orc_tensor* t = &m->t[tid];
+        if (!t->rows || orc_is_gain(tid)) continue;
+        long n = t->rows * t->cols;
+#pragma omp parallel for schedule(static)
+        for (long e = 0; e < n; e++) orc_w_store(t, e, std * orc_normal(seed, (uint64_t)tid, (uint64_t)e), m->cfg.bf16);
+    }
+}
+
+/* Planted weights for special-case tests: values are rounded to the storage precision. */
+int orc_set_tensor(orc_model* m, int tid, const double* v, long n) {
+    if (tid < 0 || tid >= m->n_tensors || !orc_tid_valid(&m->cfg, tid)) return ORC_EINVAL;
+    orc_tensor* t = &m->t[tid];
+    if (n != t->rows * t->cols) return ORC_EINVAL;
+    for (long i = 0; i < n; i++) {
+        if (orc_is_gain(tid)) t->f32[i] = (float)v[i];
+        else orc_w_store(t, i, v[i], m->cfg.bf16);
+    }
+    return ORC_OK;
+}
+
+int orc_get_tensor(const orc_model* m, int tid, long start, long count, double* out) {
+    if (tid < 0 || tid >= m->n_tensors || !orc_tid_valid(&m->cfg, tid)) return ORC_EINVAL;
+    const orc_tensor* t = &m->t[tid];
+    if (start < 0 || count < 0 || start + count > t->rows * t->cols) return ORC_EINVAL;
+    for (long i = 0; i < count; i++) out[i] = orc_w(t, start + i);
+    return ORC_OK;
+}
+
+static const orc_tensor* orc_layer_t(const orc_model* m, int l, int w) {
+    return &m->t[ORC_LAYER_BASE + ORC_LAYER_STRIDE * l + w];
+}
+
+/* ------------------------------------------------------------------------------------------
+ * Building blocks (each exported so the tests can pin it on its own).
+ * ---------------------------------------------------------------------------------------- */
+
+/* RMSNorm: y = x / sqrt(mean(x^2) + eps) * gain. */
+void orc_rmsnorm(int d, const double* x, const double* gain, double eps, double* y) {
+    double ss = 0.0;
+    for (int i = 0; i < d; i++) ss += x[i] * x[i];
+    double r = 1.0 / sqrt(ss / d + eps);
+    for (int i = 0; i < d; i++) y[i] = x[i] * r * gain[i];
+}
+
+/* Rotary embedding, rotate-half pairing (i, i + hd/2), frequency theta^(-2i/hd),
+ * angle = absolute position * frequency. In place on one head vector. */
+void orc_rope(int hd, double theta, long pos, double* v) {
+    int h = hd / 2;
+    for (int i = 0; i < h; i++) {
+        double inv = pow(theta, -(2.0 * i) / (double)hd);
+        double ang = (double)pos * inv;
+        double c = cos(ang), s = sin(ang);
+        double x1 = v[i], x2 = v[i + h];
+        v[i] = x1 * c - x2 * s;
+        v[i + h] = x2 * c + x1 * s;
+    }
+}
+
+double orc_silu(double x) { return x / (1.0 + exp(-x)); }
+
+/* y[m][n] = sum_k x[m][k] W[n][k] with W given as a double matrix (tests) */
+void orc_linear_f64(int M, int N, int K, const double* x, const double* W, double* y) {
+#pragma omp parallel for schedule(static)
+    for (long n = 0; n < N; n++)
+        for (int m = 0; m < M; m++) {
+            double acc = 0.0;
+            for (int k = 0; k < K; k++) acc += x[(long)m * K + k] * W[n * (long)K + k];
+            y[(long)m * N + n] = acc;
+        }
+}
+
+/* y[m][n] = sum_k x[m][k] W[n][k] with W a model tensor [N, K] */
+static void orc_linear_t(int M, const double* x, const orc_tensor* W, double* y) {
+    long N = W->rows, K = W->cols;
+#pragma omp parallel
+    {
+        double* wrow = (double*)malloc((size_t)K * sizeof(double));
+#pragma omp for schedule(static)
+        for (long n = 0; n < N; n++) {
+            for (long k = 0; k < K; k++) wrow[k] = orc_w(W, n * K + k);
+            for (int m = 0; m < M; m++) {
+                const double* xr = x + (long)m * K;
+                double acc = 0.0;
+                for (long k = 0; k < K; k++) acc += xr[k] * wrow[k];
+                y[(long)m * N + n] = acc;
+            }
+        }
+        free(wrow);
+    }
+}
+
+/* Grouped-query attention for one query token.
+ * q: [Hq][hd]; keys/values: n_keys entries, entry j at kptr[j] / vptr[j], each [Hkv][hd];
+ * visible[j] != 0 selects the keys this token may attend to. Query head h reads KV head
+ * h / (Hq / Hkv). Scores are scaled by 1/sqrt(hd); softmax over the visible keys.
+ * out: [Hq][hd]. A token with no visible key gets zeros. */
+void orc_attend(int Hq, int Hkv, int hd, int n_keys, const double* q, const double* const* kptr,
+                const double* const* vptr, const unsigned char* visible, double* out) {
+    int group = Hq / Hkv;
+    double scale = 1.0 / sqrt((double)hd);
+    double* s = (double*)malloc((size_t)(n_keys > 0 ? n_keys : 1) * sizeof(double));
+    for (int h = 0; h < Hq; h++) {
+        int kvh = h / group;
+        const double* qh = q + (long)h * hd;
+        double mx = -INFINITY;
+        for (int j = 0; j < n_keys; j++) {
+            if (!visible[j]) continue;
+            const double* kj = kptr[j] + (long)kvh * hd;
+            double dot = 0.0;
+            for (int i = 0; i < hd; i++) dot += qh[i] * kj[i];
+            s[j] = dot * scale;
+            if (s[j] > mx) mx = s[j];
+        }
+        double* oh = out + (long)h * hd;
+        for (int i = 0; i < hd; i++) oh[i] = 0.0;
+        if (mx == -INFINITY) continue;
+        double den = 0.0;
+        for (int j = 0; j < n_keys; j++) {
+            if (!visible[j]) continue;
+            double p = exp(s[j] - mx);
+            den += p;
+            const double* vj = vptr[j] + (long)kvh * hd;
+            for (int i = 0; i < hd; i++) oh[i] += p * vj[i];
+        }
+        for (int i = 0; i < hd; i++) oh[i] /= den;
+    }
+    free(s);
+}
+
+/* Greedy decision of Algorithm 1: argmax over the fp32-rounded logits, lowest id on ties.
+ * top2[0] = largest value, top2[1] = largest value among the other ids (fp32). */
+int orc_argmax_f32(int V, const double* logits, float* top2) {
+    int best = 0;
+    float b1 = (float)logits[0], b2 = -INFINITY;
+    for (int v = 1; v < V; v++) {
+        float x = (float)logits[v];
+        if (x > b1) { b2 = b1; b1 = x; best = v; }
+        else if (x > b2) b2 = x;
+    }
+    if (top2) { top2[0] = b1; top2[1] = b2; }
+    return best;
+}
+
+/* ------------------------------------------------------------------------------------------
+ * KV cache of one sequence: committed entries [L][max_ctx][Hkv][hd] and the in-flight K/V of
+ * the last forward [L][max_rows][Hkv][hd] (values already at the model's KV precision).
+ * ---------------------------------------------------------------------------------------- */
+typedef struct {
+    int L, Hkv, hd, max_ctx, max_rows, len;
+    double *k, *v, *sk, *sv;
+} orc_cache;
+
+void orc_cache_free(orc_cache* c) {
+    if (!c) return;
+    free(c->k); free(c->v); free(c->sk); free(c->sv);
+    free(c);
+}
+
+orc_cache* orc_cache_create(const orc_model* m, int max_ctx, int max_rows) {
+    orc_cache* c = (orc_cache*)calloc(1, sizeof(orc_cache));
+    if (!c) return NULL;
+    c->L = m->cfg.n_layers; c->Hkv = m->cfg.n_kv_heads; c->hd = m->cfg.head_dim;
+    c->max_ctx = max_ctx; c->max_rows = max_rows; c->len = 0;
+    size_t per = (size_t)c->Hkv * c->hd;
+    c->k = (double*)calloc((size_t)c->L * max_ctx * per, sizeof(double));
+    c->v = (double*)calloc((size_t)c->L * max_ctx * per, sizeof(double));
+    c->sk = (double*)calloc((size_t)c->L * max_rows * per, sizeof(double));
+    c->sv = (double*)calloc((size_t)c->L * max_rows * per, sizeof(double));
+    if (!c->k || !c->v || !c->sk || !c->sv) { orc_cache_free(c); return NULL; }
+    return c;
+}
+
+int orc_cache_len(const orc_cache* c) { return c->len; }
+
+int orc_cache_truncate(orc_cache* c, int len) {
+    if (len < 0 || len > c->len) return ORC_EINVAL;
+    c->len = len;
+    return ORC_OK;
+}
+
+/* KV commit / cache trim of Algorithm 1: the in-flight rows rows[0..n) of the last forward
+ * become cache entries len .. len+n-1, in that order. */
+int orc_commit(orc_cache* c, int n, const int32_t* rows) {
+    if (n < 0 || c->len + n > c->max_ctx) return ORC_EINVAL;
+    size_t per = (size_t)c->Hkv * c->hd;
+    for (int l = 0; l < c->L; l++)
+        for (int t = 0; t < n; t++) {
+            if (rows[t] < 0 || rows[t] >= c->max_rows) return ORC_EINVAL;
+            size_t dst = ((size_t)l * c->max_ctx + c->len + t) * per;
+            size_t src = ((size_t)l * c->max_rows + rows[t]) * per;
+            memcpy(c->k + dst, c->sk + src, per * sizeof(double));
+            memcpy(c->v + dst, c->sv + src, per * sizeof(double));
+        }
+    c->len += n;
+    return ORC_OK;
+}
+
+/* Read one K (which=0) or V (which=1) entry [Hkv][hd] of the committed cache. */
+int orc_cache_entry(const orc_cache* c, int layer, int which, int p, double* out) {
+    if (layer < 0 || layer >= c->L || p < 0 || p >= c->len) return ORC_EINVAL;
+    size_t per = (size_t)c->Hkv * c->hd;
+    const double* src = (which ? c->v : c->k) + ((size_t)layer * c->max_ctx + p) * per;
+    memcpy(out, src, per * sizeof(double));
+    return ORC_OK;
+}
+
+/* ------------------------------------------------------------------------------------------
+ * One forward pass over M in-flight rows (Eq. 3 with the mask of Sec. 3.2 / Algorithm 1).
+ * Row i carries token tokens[i] at absolute position pos[i] and belongs to segment seg[i].
+ * Row i attends to every committed cache entry (positions 0 .. len-1) and to in-flight row j
+ * iff seg[j] == seg[i] and pos[j] <= pos[i] (causal inside a segment), or segment seg[j] is
+ * an ancestor of seg[i] (bit seg[j] of anc[seg[i]]). The in-flight K/V of every row is kept
+ * for a later orc_commit. Outputs: argmax[M]; optional fp32 top-2 [M][2]; optional fp64
+ * logits [M][V]; optional final hidden state [M][d] (before the final norm).
+ * ---------------------------------------------------------------------------------------- */
+int orc_forward(const orc_model* m, orc_cache* c, int M, const int32_t* tokens, const int32_t* pos,
+                const int32_t* seg, const uint32_t* anc, int n_seg, int32_t* argmax_out,
+                float* top2_out, double* logits_out, double* hidden_out) {
+    const orc_config* cf = &m->cfg;
+    int d = cf->d_model, Hq = cf->n_heads, Hkv = cf->n_kv_heads, hd = cf->head_dim, F = cf->d_ff,
+        V = cf->vocab, L = cf->n_layers;
+    int qd = Hq * hd, kvd = Hkv * hd;
+    int bf = cf->bf16;
+    if (M < 1 || M > c->max_rows || n_seg < 1 || n_seg > 32) return ORC_EINVAL;
+    for (int i = 0; i < M; i++) {
+        if (tokens[i] < 0 || tokens[i] >= V || seg[i] < 0 || seg[i] >= n_seg || pos[i] < c->len ||
+            pos[i] >= c->max_ctx)
+            return ORC_EINVAL;
+    }
+#define RB(x) (bf ? orc_round_bf16(x) : (x))
+    double* x = (double*)calloc((size_t)M * d, sizeof(double));
+    double* h = (double*)calloc((size_t)M * d, sizeof(double));
+    double* q = (double*)calloc((size_t)M * qd, sizeof(double));
+    double* kk = (double*)calloc((size_t)M * kvd, sizeof(double));
+    double* vv = (double*)calloc((size_t)M * kvd, sizeof(double));
+    double* att = (double*)calloc((size_t)M * qd, sizeof(double));
+    double* tmp = (double*)calloc((size_t)M * (d > qd ? d : qd), sizeof(double));
+    double* gt = (double*)calloc((size_t)M * F, sizeof(double));
+    double* ut = (double*)calloc((size_t)M * F, sizeof(double));
+    double* gain = (double*)calloc((size_t)d, sizeof(double));
+    if (!x || !h || !q || !kk || !vv || !att || !tmp || !gt || !ut || !gain) {
+        free(x); free(h); free(q); free(kk); free(vv); free(att); free(tmp); free(gt); free(ut); free(gain);
+        return ORC_ENOMEM;
+    }
+    /* embedding lookup */
+    for (int i = 0; i < M; i++)
+        for (int j = 0; j < d; j++) x[(long)i * d + j] = orc_w(&m->t[T_EMBED], (long)tokens[i] * d + j);
+
+    size_t per = (size_t)kvd;
+    for (int l = 0; l < L; l++) {
+        /* attention block */
+        for (int j = 0; j < d; j++) gain[j] = orc_w(orc_layer_t(m, l, L_ANORM), j);
+        for (int i = 0; i < M; i++) {
+            orc_rmsnorm(d, x + (long)i * d, gain, cf->rms_eps, h + (long)i * d);
+            for (int j = 0; j < d; j++) h[(long)i * d + j] = RB(h[(long)i * d + j]);
+        }
+        orc_linear_t(M, h, orc_layer_t(m, l, L_WQ), q);
+        orc_linear_t(M, h, orc_layer_t(m, l, L_WK), kk);
+        orc_linear_t(M, h, orc_layer_t(m, l, L_WV), vv);
+        for (int i = 0; i < M; i++) {
+            for (int hh = 0; hh < Hq; hh++) orc_rope(hd, cf->rope_theta, pos[i], q + (long)i * qd + (long)hh * hd);
+            for (int hh = 0; hh < Hkv; hh++) orc_rope(hd, cf->rope_theta, pos[i], kk + (long)i * kvd + (long)hh * hd);
+            for (int j = 0; j < qd; j++) q[(long)i * qd + j] = RB(q[(long)i * qd + j]);
+            for (int j = 0; j < kvd; j++) {
+                kk[(long)i * kvd + j] = RB(kk[(long)i * kvd + j]);
+                vv[(long)i * kvd + j] = RB(vv[(long)i * kvd + j]);
+            }
+            memcpy(c->sk + ((size_t)l * c->max_rows + i) * per, kk + (long)i * kvd, per * sizeof(double));
+            memcpy(c->sv + ((size_t)l * c->max_rows + i) * per, vv + (long)i * kvd, per * sizeof(double));
+        }
+        int nk = c->len + M;
+#pragma omp parallel
+        {
+            const double** kp = (const double**)malloc((size_t)nk * sizeof(double*));
+            const double** vp = (const double**)malloc((size_t)nk * sizeof(double*));
+            unsigned char* vis = (unsigned char*)malloc((size_t)nk);
+#pragma omp for schedule(dynamic, 1)
+            for (int i = 0; i < M; i++) {
+                for (int j = 0; j < c->len; j++) {
+                    kp[j] = c->k + ((size_t)l * c->max_ctx + j) * per;
+                    vp[j] = c->v + ((size_t)l * c->max_ctx + j) * per;
+                    vis[j] = 1;
+                }
+                for (int j = 0; j < M; j++) {
+                    int jj = c->len + j;
+                    kp[jj] = kk + (long)j * kvd;
+                    vp[jj] = vv + (long)j * kvd;
+                    int same = (seg[j] == seg[i]) && (pos[j] <= pos[i]);
+                    int ancestor = (seg[j] != seg[i]) && ((anc[seg[i]] >> seg[j]) & 1u);
+                    vis[jj] = (unsigned char)(same || ancestor);
+                }
+                orc_attend(Hq, Hkv, hd, nk, q + (long)i * qd, kp, vp, vis, att + (long)i * qd);
+            }
+            free(kp); free(vp); free(vis);
+        }
+        for (long j = 0; j < (long)M * qd; j++) att[j] = RB(att[j]);
+        orc_linear_t(M, att, orc_layer_t(m, l, L_WO), tmp);
+        for (long j = 0; j < (long)M * d; j++) x[j] += tmp[j];
+
+        /* MLP block */
+        for (int j = 0; j < d; j++) gain[j] = orc_w(orc_layer_t(m, l, L_MNORM), j);
+        for (int i = 0; i < M; i++) {
+            orc_rmsnorm(d, x + (long)i * d, gain, cf->rms_eps, h + (long)i * d);
+            for (int j = 0; j < d; j++) h[(long)i * d + j] = RB(h[(long)i * d + j]);
+        }
+        orc_linear_t(M, h, orc_layer_t(m, l, L_WG), gt);
+        orc_linear_t(M, h, orc_layer_t(m, l, L_WU), ut);
+        for (long j = 0; j < (long)M * F; j++) gt[j] = RB(orc_silu(gt[j]) * ut[j]);
+        orc_linear_t(M, gt, orc_layer_t(m, l, L_WD), tmp);
+        for (long j = 0; j < (long)M * d; j++) x[j] += tmp[j];
+    }
+    if (hidden_out) memcpy(hidden_out, x, (size_t)M * d * sizeof(double));
+
+    /* final norm, LM head, greedy decision */
+    for (int j = 0; j < d; j++) gain[j] = orc_w(&m->t[T_FNORM], j);
+    for (int i = 0; i < M; i++) {
+        orc_rmsnorm(d, x + (long)i * d, gain, cf->rms_eps, h + (long)i * d);
+        for (int j = 0; j < d; j++) h[(long)i * d + j] = RB(h[(long)i * d + j]);
+    }
+    free(gt); gt = NULL;
+    double* logits = (double*)malloc((size_t)M * V * sizeof(double));
+    if (!logits) {
+        free(x); free(h); free(q); free(kk); free(vv); free(att); free(tmp); free(ut); free(gain);
+        return ORC_ENOMEM;
+    }
+    orc_linear_t(M, h, &m->t[T_LMHEAD], logits);
+    for (int i = 0; i < M; i++) {
+        int a = orc_argmax_f32(V, logits + (long)i * V, top2_out ? top2_out + 2 * i : NULL);
+        if (argmax_out) argmax_out[i] = a;
+    }
+    if (logits_out) memcpy(logits_out, logits, (size_t)M * V * sizeof(double));
+#undef RB
+    free(logits); free(x); free(h); free(q); free(kk); free(vv); free(att); free(tmp); free(ut); free(gain);
+    return ORC_OK;
+}
+
+int orc_num_threads(void) {
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
+
+void orc_set_num_threads(int n) {
+#ifdef _OPENMP
+    if (n > 0) omp_set_num_threads(n);
+#else
+    (void)n;
+#endif
+}

@@ -1,0 +1,319 @@
+"""Benchmark of the Jacobi-decoding hot path on GB300: committed tokens/s on the Qwen2.5-7B-shaped
+bf16 decoder at batch 1 (prompt 1024, block n = 32, 512 new tokens, draft injection p = 0.3
+against the model's own greedy continuation, paged KV with 16-token pages).
+
+One step = one jf_generate_device call: prefill of the prompt plus every Jacobi iteration until
+512 new tokens are committed. Inputs are resident on the device when the timed region starts
+(`value`); `e2e` repeats the measurement through jf_generate with host buffers (prompt and truth
+copied in, tokens copied out inside the timed region).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference] [--no-cpu-baseline]
+
+For N > 1 (torchrun) every rank runs an independent replica of the workload (the path does not
+shard); value = tokens of all ranks / max-over-ranks time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "tokens/s at bs1 on 7B-shape; Jacobi-iteration latency as % of HBM roofline"
+WORKLOAD = "qwen2.5-7b-shape-bf16 prompt1024 block32 new512 inject-p0.3 paged-kv16 bs1"
+PROMPT_LEN, BLOCK, NEW, P_INJECT = 1024, 32, 512, 0.3
+NOMINAL_HBM_GBS = 8000.0
+# DRAM bytes (read + write) per launch of the gate/up projection at M = 32 rows, from the ncu capture
+# summarised in profiles/gateup_gemm_7b_m32.md; None until a capture of the current kernel exists.
+GATEUP_TRAFFIC_BYTES = None
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clocks/throttle reasons sampled during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.dev = device_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "200",
+                 "-i", str(self.dev)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.t.join(timeout=2)
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [x.strip() for x in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[5:9]):
+                if v.lower() in ("active", "1", "0x1"):
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------------------------------------------
+# CPU oracle sample (the reference arm and the cpu_baseline object)
+# ------------------------------------------------------------------------------------------
+def oracle_sample(steps: int, warmup: int):
+    """Jacobi iterations of the oracle on the same 7B-shaped model and block size, with the
+    prompt cut to its first 16 tokens (the oracle cannot prefill 1024 tokens in minutes)."""
+    from oracle import jacobi as OJ
+    from oracle import oracle as O
+    from paper_2512_14681_gb300 import inputs as I
+
+    shape = I.QWEN7B_BF16
+    need = shape.weight_bytes() + (6 << 30)
+    avail = os.sysconf("SC_AVPHYS_PAGES") * os.sysconf("SC_PAGE_SIZE")
+    if avail < need:
+        return None, f"host memory {avail >> 30} GiB < {need >> 30} GiB needed by the 7B oracle"
+    prompt = I.prompt_tokens(shape.vocab, PROMPT_LEN)[:16]
+    model = O.Model(O.ModelConfig(**shape.oracle_kwargs())).init_random(I.WEIGHT_SEED, I.WEIGHT_STD)
+    n_it = steps + warmup
+    truth = OJ.generate_ar(model, prompt, n_it * BLOCK + 2 * BLOCK + 2).tokens
+    dec = OJ.JacobiDecoder(model, prompt, OJ.GenParams(block_size=BLOCK, init="inject", inject_p=P_INJECT,
+                                                       seed=I.INJECT_SEED, max_new=len(truth) - 2 * BLOCK - 2),
+                           truth=truth)
+    for _ in range(warmup):
+        dec.step()
+    t0 = time.perf_counter()
+    toks = 0
+    for _ in range(steps):
+        toks += dec.step().k
+    dt = time.perf_counter() - t0
+    return dict(value=toks / dt, unit="tokens/s", cores=O.num_threads(), kind="oracle",
+                sample=f"{steps} Jacobi iterations (n={BLOCK}, inject p={P_INJECT}) of the 7B-shaped model "
+                       f"after a 16-token prompt prefill; {toks} tokens in {dt:.1f} s"), None
+
+
+def run_reference(args, rank):
+    if rank != 0:
+        return
+    res, why = oracle_sample(args.steps, args.warmup)
+    if res is None:
+        print(json.dumps({"impl": "reference", "unavailable": why}))
+        return
+    line = {"impl": "reference", "metric": METRIC, "value": res["value"], "unit": "tokens/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 * 1.0 / max(res["value"], 1e-9),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": WORKLOAD, "sample": res["sample"]},
+            "cpu_baseline": res, "e2e": {"value": res["value"], "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                                         "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+
+
+# ------------------------------------------------------------------------------------------
+# GPU arm
+# ------------------------------------------------------------------------------------------
+def run_gpu(args, rank, world, local_rank):
+    import torch
+
+    from paper_2512_14681_gb300 import inputs as I
+    from paper_2512_14681_gb300.jacobi import Context, Gen
+
+    torch.cuda.set_device(local_rank)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    shape = I.QWEN7B_BF16
+    truth_len = NEW + 2 * BLOCK + 1
+    # max_rows 512: the 1024-token prompt is prefilled in two 512-row forwards
+    ctx = Context(shape, max_seqs=1, max_ctx=2048, max_rows=512)
+    ctx.init_random_weights(I.WEIGHT_SEED, I.WEIGHT_STD)
+    prompt = I.prompt_tokens(shape.vocab, PROMPT_LEN)
+    truth = ctx.generate([prompt], Gen(mode="ar", max_new=truth_len)).tokens[0].astype(np.int32)
+    gen = Gen(block_size=BLOCK, init="inject", inject_p=P_INJECT, seed=I.INJECT_SEED, max_new=NEW)
+    d_prompt = torch.from_numpy(prompt).cuda()
+    d_truth = torch.from_numpy(truth).cuda().reshape(1, -1)
+    d_out = torch.empty((1, NEW), dtype=torch.int32, device="cuda")
+    st = ctx.stream
+
+    def step(log_cap=0):
+        return ctx.generate_device(d_prompt, [PROMPT_LEN], gen, d_out, d_truth, truth_len, log_cap=log_cap)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    first = step(log_cap=1024)
+    assert np.array_equal(d_out.cpu().numpy()[0], truth[:NEW]), "generated tokens differ from the greedy truth"
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    # ---- timed region: device-resident inputs
+    sampler = ClockSampler(local_rank)
+    barrier()
+    sampler.start()
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    ev0.record(st)
+    launches = 0
+    iters = 0
+    decode_ms = 0.0
+    prefill_ms = 0.0
+    for _ in range(args.steps):
+        o = step()
+        launches += o.kernel_launches
+        iters += o.iterations
+        decode_ms += o.decode_ms
+        prefill_ms += o.prefill_ms
+    ev1.record(st)
+    barrier()
+    clocks = sampler.stop()
+    total_ms = ev0.elapsed_time(ev1)
+    if dist is not None:
+        t = torch.tensor([total_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    ms_per_step = total_ms / args.steps
+    value = world * NEW * args.steps / (total_ms / 1000.0)
+
+    # ---- end to end: host buffers in and out through jf_generate
+    barrier()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(st)
+    for _ in range(args.steps):
+        h = ctx.generate([prompt], gen, truth=truth.reshape(1, -1), log_cap=0)
+    e1.record(st)
+    barrier()
+    e2e_ms = e0.elapsed_time(e1)
+    assert np.array_equal(h.tokens[0], truth[:NEW])
+    e2e_value = world * NEW * args.steps / (e2e_ms / 1000.0)
+
+    # ---- per-kernel timing of the dominant kernel (CUDA events around its launches)
+    ctx.set_profiling(True)
+    for _ in range(max(1, min(args.steps, 2))):
+        step()
+    torch.cuda.synchronize()
+    gu_ms, gu_n = ctx.kernel_time(0)
+    at_ms, at_n = ctx.kernel_time(1)
+    ctx.set_profiling(False)
+
+    if rank != 0:
+        if dist is not None:
+            dist.destroy_process_group()
+        return
+    peak, peak_kind = _peaks()
+    rows = first.rows.astype(np.float64)
+    m_avg = float(rows.mean()) if rows.size else float(BLOCK)
+    d, F = shape.d_model, shape.d_ff
+    gu_bytes = 2 * F * d * 2 + m_avg * d * 2 + m_avg * F * 2
+    gu_avg_s = gu_ms / max(gu_n, 1) / 1000.0
+    achieved = gu_bytes / gu_avg_s / 1e9 if gu_n else None
+    # per-iteration roofline: every weight byte + the committed KV read once per iteration
+    n_iter = first.iterations
+    it_ms = first.decode_ms / max(n_iter, 1)
+    kv_tok = shape.kv_bytes_per_token()
+    p_avg = PROMPT_LEN + NEW / 2.0
+    it_bytes = shape.weight_bytes() + kv_tok * p_avg
+    it_gbs = it_bytes / (it_ms / 1000.0) / 1e9
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic: uniform-random prompt, N(0,0.02) random weights, drafts injected from the model's own "
+                "greedy continuation",
+        "config": {"workload": WORKLOAD, "prompt": PROMPT_LEN, "block_size": BLOCK, "new_tokens": NEW,
+                   "inject_p": P_INJECT, "kv_page_tokens": 16, "batch": 1,
+                   "parallelism": "replicas" if world > 1 else "single-gpu",
+                   "l2": "no flush: every step streams 14.1 GB of weights through the 129 MB L2"},
+        "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": int(prompt.nbytes + truth.nbytes),
+                "d2h_bytes_per_step": int(NEW * 4)},
+        "gpu_launches": int(launches),
+        "iteration": {"count_per_step": n_iter, "tokens_per_iteration": NEW / max(n_iter, 1), "ms": it_ms,
+                      "prefill_ms": first.prefill_ms, "bytes": it_bytes, "achieved_gbs": it_gbs,
+                      "frac_of_" + peak_kind: it_gbs / peak, "frac_of_8tbs": it_gbs / NOMINAL_HBM_GBS},
+        "roofline": {"bound": "hbm", "kernel": "gate/up projection GEMM (tcgen05, SwiGLU epilogue)",
+                     "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": (achieved / peak) if achieved else None, "traffic": GATEUP_TRAFFIC_BYTES,
+                     "bytes_per_launch": gu_bytes, "launches_timed": gu_n, "avg_launch_us": gu_avg_s * 1e6,
+                     "peak_kind": peak_kind, "timing": "CUDA events around each launch in a profiled pass of the step"},
+        "attention": {"launches_timed": at_n, "avg_launch_us": (at_ms / max(at_n, 1)) * 1000.0},
+        "clocks": clocks,
+    }
+    if args.cpu_baseline and world == 1:
+        cb, why = oracle_sample(args.cpu_baseline_iters, 0)
+        line["cpu_baseline"] = cb if cb is not None else {"unavailable": why}
+    else:
+        line["cpu_baseline"] = None
+    print(json.dumps(line))
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
+    ap.add_argument("--cpu-baseline-iters", type=int, default=2)
+    args = ap.parse_args()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank)
+        return
+    import __graft_entry__
+
+    __graft_entry__.build()
+    run_gpu(args, rank, world, local_rank)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,193 @@
+/*
+ * jf.h -- C ABI of libjf: the Jacobi-decoding hot path of Jacobi Forcing (arXiv 2512.14681)
+ * on one NVIDIA GB300 (sm_103a).
+ *
+ * One Jacobi iteration (Sec. 2.1, Eq. 3; Sec. 3.2 and Algorithm 1 for multi-block decoding and
+ * rejection recycling) runs a block of n draft tokens -- or K blocks plus recycled candidates --
+ * through ONE forward pass of a causal decoder-only transformer over the exact KV cache of the
+ * committed prefix, takes the greedy argmax of every row, accepts the longest fixed-point prefix
+ * of the real-active draft (its first token is always correct) and commits that prefix's K/V.
+ *
+ * Conventions shared by every call:
+ *   - Plain pointers and sizes only. "host" pointers are CPU memory, "device" pointers are GPU
+ *     memory of the context's device. The caller owns every buffer it passes; the library never
+ *     frees caller memory and keeps no pointer to a host buffer after the call returns.
+ *   - Device memory: the caller allocates ONE arena of jf_arena_bytes() bytes (e.g. through
+ *     PyTorch) and lends it to the context until jf_destroy(). The library allocates no device
+ *     memory of its own; it allocates small pinned host buffers for per-iteration results.
+ *   - Work is ordered on the caller's CUDA stream (jf_runtime_config.cuda_stream; NULL lets the
+ *     library create a non-blocking stream). Calls that return host outputs synchronise it.
+ *   - Every call returns a jf_status. Arguments are validated on the host before any launch; a
+ *     call that fails validation changes no state. jf_last_error() returns a message for the last
+ *     failure. A context is not thread-safe.
+ *   - Device-side checks (index bounds, bounded waits of the tensor-core pipeline) report through
+ *     an error word read back after each call: JF_EDEVICE / JF_ETIMEOUT. No kernel traps.
+ */
+#ifndef JF_H
+#define JF_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  JF_OK = 0,
+  JF_EINVAL = 1,        /* invalid argument, shape or call sequence parameter */
+  JF_ENOMEM = 2,        /* arena too small, or pinned host allocation failed */
+  JF_ECAPACITY = 3,     /* KV pages, rows, sequences or context length exhausted */
+  JF_ESTATE = 4,        /* call out of order (e.g. step before prefill, no weights) */
+  JF_EIO = 5,           /* weight file missing, truncated or of another shape */
+  JF_ECUDA = 6,         /* a CUDA runtime call failed */
+  JF_EDEVICE = 7,       /* a kernel found an out-of-range index (bounds check) */
+  JF_ETIMEOUT = 8,      /* a bounded device wait gave up */
+  JF_EUNSUPPORTED = 9   /* shape not supported by the kernels (see jf_create) */
+} jf_status;
+
+typedef enum { JF_F32 = 0, JF_BF16 = 1 } jf_dtype;
+
+/* Decoder shape (Sec. 4.1: the Qwen2.5 family). RMSNorm -> fused QKV -> rotary embedding
+ * (rotate-half pairing, frequency rope_theta^(-2i/head_dim)) -> grouped-query attention ->
+ * O projection + residual -> RMSNorm -> SwiGLU MLP + residual; final RMSNorm -> LM head.
+ * dtype JF_BF16: weights, KV cache and matrix-product inputs are bf16; accumulation, residual
+ * stream, softmax and logits are fp32. JF_F32: everything fp32 (CUDA-core kernels).
+ * Supported: head_dim 128 (bf16) or 64/128 (fp32); n_heads*head_dim and n_kv_heads*head_dim
+ * multiples of 128; d_model and d_ff multiples of 64; n_heads a multiple of n_kv_heads. */
+typedef struct {
+  int n_layers, d_model, n_heads, n_kv_heads, head_dim, d_ff, vocab;
+  double rms_eps, rope_theta;
+  int dtype;
+} jf_model_config;
+
+/* Capacity. max_rows: in-flight rows per forward (K*n + candidates, or a prefill chunk);
+ * max_ctx: positions per sequence (KV pages of 16 tokens are reserved for it);
+ * logits_rows: rows jf_forward_logits() may return (0 = that call is unavailable). */
+typedef struct {
+  int max_seqs, max_ctx, max_rows, logits_rows;
+  void* device_arena;
+  size_t arena_bytes;
+  void* cuda_stream;
+} jf_runtime_config;
+
+typedef struct jf_ctx jf_ctx;
+
+/* Bytes of device arena a context of this shape needs (host-only, no GPU work). */
+jf_status jf_arena_bytes(const jf_model_config* model, const jf_runtime_config* rt, size_t* out_bytes);
+
+/* Create a context on the current CUDA device; carves the arena, builds the rotary table. */
+jf_status jf_create(const jf_model_config* model, const jf_runtime_config* rt, jf_ctx** out);
+void jf_destroy(jf_ctx* ctx);
+const char* jf_last_error(const jf_ctx* ctx);
+
+/* Weights. Logical tensors, row-major [out, in]: id 0 embedding [V,d], 1 LM head [V,d],
+ * 2 final-norm gain [d]; layer l at 8+16l: +0 attention-norm gain [d], +1 Wq [Hq*hd,d],
+ * +2 Wk [Hkv*hd,d], +3 Wv [Hkv*hd,d], +4 Wo [d,Hq*hd], +5 MLP-norm gain [d], +6 W_gate [F,d],
+ * +7 W_up [F,d], +8 W_down [d,F].
+ * jf_init_random_weights: every matrix entry = std * N(0,1) from SplitMix64 + Box-Muller keyed
+ * by (seed, tensor id, element index), rounded to the model dtype; gains = 1.
+ * jf_load_weights / jf_save_weights: raw file "JFW1" (header with the shape, then the tensors in
+ * id order, matrices in the model dtype, gains fp32).
+ * jf_get_weights: copies `count` logical elements of tensor `tensor_id` from `start` into a host
+ * fp32 buffer. */
+jf_status jf_init_random_weights(jf_ctx* ctx, uint64_t seed, double std);
+jf_status jf_load_weights(jf_ctx* ctx, const char* path);
+jf_status jf_save_weights(jf_ctx* ctx, const char* path);
+jf_status jf_get_weights(jf_ctx* ctx, int tensor_id, long long start, long long count, float* out_host);
+
+/* Prefill (Eq. 1 context x): commit the K/V of `len` prompt tokens (host array) after the
+ * sequence's current length, in chunks of max_rows; *next_token (host) = greedy argmax after the
+ * last prompt token, i.e. the known-correct first token q0 of the first Jacobi block. */
+jf_status jf_prefill(jf_ctx* ctx, int seq, const int32_t* prompt, int len, int32_t* next_token);
+jf_status jf_truncate(jf_ctx* ctx, int seq, int len);
+jf_status jf_seq_len(jf_ctx* ctx, int seq, int* out_len);
+
+/* One block of a Jacobi step. kind: JF_BLOCK_RA (the real-active draft; exactly one, starting
+ * at the committed length P, first token = the known-correct q0), JF_BLOCK_PSEUDO (a
+ * pseudo-active block that continues the previous RA/pseudo block: start_pos = its end,
+ * parent = its index), JF_BLOCK_CAND (a recycled candidate: start_pos = P, parent = -1). */
+typedef enum { JF_BLOCK_RA = 0, JF_BLOCK_PSEUDO = 1, JF_BLOCK_CAND = 2 } jf_block_kind;
+typedef struct {
+  int kind, start_pos, len, parent;
+} jf_block;
+
+/* One Jacobi iteration of sequence `seq` with caller-supplied blocks (Eq. 3; Algorithm 1
+ * assemble / forward / verify / cache trim). draft_tokens: host, sum(len) tokens, blocks in
+ * order. Outputs (host): accepted_counts[n_blocks] (RA/candidate: 1 + longest run of draft
+ * tokens equal to the prediction of the row before them; pseudo: the same run with no free
+ * first token); committed_tokens[<= max len] and *n_committed: the winning draft's accepted
+ * prefix (largest count, ties to the RA block), whose K/V is committed; predictions[sum(len)]
+ * (optional): greedy argmax of every row; top2[sum(len)][2] (optional): fp32 largest and
+ * second-largest logit of every row. */
+jf_status jf_jacobi_step(jf_ctx* ctx, int seq, int n_blocks, const jf_block* blocks, const int32_t* draft_tokens,
+                         int32_t* accepted_counts, int32_t* committed_tokens, int32_t* n_committed,
+                         int32_t* predictions, float* top2);
+
+/* Forward of `n_rows` tokens (host) of sequence `seq` at positions P .. P+n_rows-1 with a causal
+ * mask, WITHOUT committing: fp32 logits [n_rows][V], final residual stream [n_rows][d] (before
+ * the final norm) and argmax [n_rows], each optional (host). n_rows <= logits_rows. */
+jf_status jf_forward_logits(jf_ctx* ctx, int seq, int n_rows, const int32_t* tokens, float* logits, float* hidden,
+                            int32_t* argmax);
+
+typedef enum { JF_MODE_BLOCK = 0, JF_MODE_WINDOW = 1, JF_MODE_AR = 2 } jf_gen_mode;
+typedef enum { JF_INIT_REPEAT = 0, JF_INIT_INJECT = 1 } jf_gen_init;
+
+/* Generation parameters (Eq. 4 block-sequential decoding; running window, Sec. 4.2; Algorithm 1).
+ * block_size n; n_blocks K (1 = single block; K > 1 needs JF_MODE_BLOCK); spawn_ratio r (a
+ * pseudo block is spawned while fewer than K are active and the newest block has >= ceil(r n)
+ * accepted tokens); pool_size / ngram_len G (0 = n) / cand_per_iter: rejection-recycling pool
+ * of rejected real-active tails and candidates verified per iteration (pool_size 0 = off);
+ * init JF_INIT_REPEAT (free draft positions = the last committed token; Jacobi update
+ * thereafter) or JF_INIT_INJECT (free draft positions = truth token, replaced with probability
+ * inject_p by another uniform token, keyed by (seed, position, iteration)); truth: greedy
+ * continuation of each prompt, [n_seqs][truth_len], required for INJECT with
+ * truth_len >= max_new + n_blocks*block_size + G + 1; eos_id -1 = none. */
+typedef struct {
+  int block_size, n_blocks;
+  double spawn_ratio;
+  int pool_size, ngram_len, cand_per_iter;
+  int mode, init;
+  float inject_p;
+  uint64_t seed;
+  int max_new, eos_id;
+  const int32_t* truth;
+  int truth_len;
+} jf_gen_params;
+
+/* Statistics of one generation. accepted (optional caller buffer [accepted_cap][n_seqs]):
+ * tokens committed per iteration (-1 once a sequence is done); rows (optional [accepted_cap]):
+ * in-flight rows of each iteration. Times from CUDA events on the context's stream.
+ * kernel_launches: libjf kernels launched by the call (prefill, setup and every node of every
+ * replayed decode-iteration graph). */
+typedef struct {
+  int iterations;
+  int32_t* accepted;
+  int32_t* rows;
+  int accepted_cap;
+  double prefill_ms, decode_ms;
+  long long kernel_launches;
+} jf_gen_stats;
+
+/* Prefill then Jacobi-decode n_seqs independent sequences (slots 0 .. n_seqs-1, which are reset)
+ * until max_new tokens each (or EOS). Host buffers: prompts[i] (prompt_lens[i] tokens),
+ * params->truth, out_tokens [n_seqs][max_new] (tokens after an EOS are left as -1). */
+jf_status jf_generate(jf_ctx* ctx, int n_seqs, const int32_t* const* prompts, const int32_t* prompt_lens,
+                      const jf_gen_params* params, int32_t* out_tokens, jf_gen_stats* stats);
+
+/* Same with device buffers: d_prompts = the prompts concatenated, prompt_lens (HOST array),
+ * params->truth a DEVICE pointer [n_seqs][truth_len], d_out_tokens DEVICE [n_seqs][max_new]. */
+jf_status jf_generate_device(jf_ctx* ctx, int n_seqs, const int32_t* d_prompts, const int32_t* prompt_lens,
+                             const jf_gen_params* params, int32_t* d_out_tokens, jf_gen_stats* stats);
+
+/* Cumulative device time (ms, CUDA events) and launch count of one kernel class inside
+ * jf_generate* decode iterations, when profiling is enabled with jf_set_profiling(ctx, 1).
+ * kernel_class: 0 = gate/up projection GEMM (the largest weight stream), 1 = attention,
+ * 2 = all projection GEMMs. */
+jf_status jf_set_profiling(jf_ctx* ctx, int enable);
+jf_status jf_kernel_time(jf_ctx* ctx, int kernel_class, double* total_ms, long long* launches);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* JF_H */

@@ -1,0 +1,165 @@
+// Small kernels of the forward pass: random weights, the rotary table, embedding lookup and
+// RMSNorm (the Qwen2.5-style decoder of Sec. 4.1).
+#include "jf_device.cuh"
+#include "jf_internal.h"
+
+namespace jf {
+namespace {
+
+// SplitMix64 (Steele, Lea & Flood 2014): the i-th output of a stream started at state s.
+__device__ __forceinline__ uint64_t sm64_out(uint64_t s, uint64_t i) {
+  uint64_t z = s + (i + 1ull) * 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+// Weight tensor of `rows` x `cols` logical entries, entry e = std * N(0,1) drawn by Box-Muller
+// from outputs 2j, 2j+1 (j = e / 2) of the SplitMix64 stream keyed by output `tid` of the stream
+// seeded with `seed`. Logical row r lands at device row (r / grp) * grp_stride + r % grp + grp_off.
+template <typename T>
+__global__ void k_init_weights(T* dst, long long rows, long long cols, uint64_t seed, uint64_t tid, double stdv,
+                               long long grp, long long grp_stride, long long grp_off) {
+  const long long n = rows * cols;
+  const long long npairs = (n + 1) / 2;
+  const uint64_t s = sm64_out(seed, tid);
+  const double two53 = 9007199254740992.0;
+  for (long long j = blockIdx.x * (long long)blockDim.x + threadIdx.x; j < npairs;
+       j += (long long)gridDim.x * blockDim.x) {
+    const uint64_t a = sm64_out(s, 2ull * j), b = sm64_out(s, 2ull * j + 1);
+    const double u1 = ((double)(a >> 11) + 1.0) / two53;
+    const double u2 = (double)(b >> 11) / two53;
+    const double rad = sqrt(-2.0 * log(u1));
+    double sn, cs;
+    sincos(2.0 * 3.14159265358979323846 * u2, &sn, &cs);
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const long long e = 2 * j + h;
+      if (e >= n) break;
+      const double z = stdv * rad * (h ? sn : cs);
+      const long long r = e / cols, c = e % cols;
+      const long long dr = (r / grp) * grp_stride + (r % grp) + grp_off;
+      if constexpr (sizeof(T) == 2) dst[dr * cols + c] = __double2bfloat16(z);
+      else dst[dr * cols + c] = (float)z;
+    }
+  }
+}
+
+__global__ void k_fill_f32(float* p, long long n, float v) {
+  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x)
+    p[i] = v;
+}
+
+// (cos, sin) of position * theta^(-2i/hd), computed in fp64 and stored as fp32.
+__global__ void k_rope_table(float2* tab, int n_pos, int half, double theta) {
+  const long long n = (long long)n_pos * half;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < n; e += (long long)gridDim.x * blockDim.x) {
+    const int p = (int)(e / half), i = (int)(e % half);
+    const double inv = pow(theta, -(2.0 * i) / (2.0 * half));
+    double sn, cs;
+    sincos((double)p * inv, &sn, &cs);
+    tab[e] = make_float2((float)cs, (float)sn);
+  }
+}
+
+// x[r, :] = E[tok[r], :] (fp32 residual stream)
+template <typename T>
+__global__ void k_embed(const T* __restrict__ E, const int* __restrict__ tok, float* __restrict__ x, int d, int V,
+                        int* err) {
+  pdl_wait();
+  const int r = blockIdx.x;
+  int t = tok[r];
+  if (t < 0 || t >= V) {
+    if (threadIdx.x == 0) jf_set_error(err, JF_DERR_BOUNDS);
+    t = 0;
+  }
+  const T* src = E + (size_t)t * d;
+  float* dst = x + (size_t)r * d;
+  for (int i = threadIdx.x; i < d; i += blockDim.x) dst[i] = act_to_f32(src[i]);
+  pdl_launch_dependents();
+}
+
+// y[r, :] = x[r, :] / sqrt(mean(x[r, :]^2) + eps) * gain, rounded to the activation type.
+template <typename T>
+__global__ void __launch_bounds__(256) k_rmsnorm(const float* __restrict__ x, const float* __restrict__ gain,
+                                                 T* __restrict__ y, int d, float eps) {
+  __shared__ float red[8];
+  pdl_wait();
+  const int r = blockIdx.x;
+  const float* xr = x + (size_t)r * d;
+  float ss = 0.f;
+  for (int i = threadIdx.x; i < d; i += 256) ss = fmaf(xr[i], xr[i], ss);
+  ss = warp_sum(ss);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+  __syncthreads();
+  float tot = 0.f;
+#pragma unroll
+  for (int w = 0; w < 8; ++w) tot += red[w];
+  const float rs = 1.0f / sqrtf(tot / (float)d + eps);
+  T* yr = y + (size_t)r * d;
+  for (int i = threadIdx.x; i < d; i += 256) yr[i] = to_act<T>(xr[i] * rs * gain[i]);
+  pdl_launch_dependents();
+}
+
+template <typename K, typename... Args>
+cudaError_t launch_pdl(K kernel, dim3 grid, dim3 block, cudaStream_t st, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.stream = st;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
+}  // namespace
+
+cudaError_t launch_init_weights(void* dst, bool is_bf16, long long rows, long long cols, uint64_t seed, uint64_t tid,
+                                double stdv, long long grp, long long grp_stride, long long grp_off, cudaStream_t st) {
+  const long long npairs = (rows * cols + 1) / 2;
+  long long blocks = (npairs + 255) / 256;
+  if (blocks > 152 * 64) blocks = 152 * 64;
+  if (blocks < 1) blocks = 1;
+  if (is_bf16)
+    k_init_weights<bf16><<<(unsigned)blocks, 256, 0, st>>>(reinterpret_cast<bf16*>(dst), rows, cols, seed, tid, stdv,
+                                                           grp, grp_stride, grp_off);
+  else
+    k_init_weights<float><<<(unsigned)blocks, 256, 0, st>>>(reinterpret_cast<float*>(dst), rows, cols, seed, tid,
+                                                            stdv, grp, grp_stride, grp_off);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_fill_f32(float* p, long long n, float v, cudaStream_t st) {
+  long long blocks = (n + 255) / 256;
+  if (blocks > 4096) blocks = 4096;
+  if (blocks < 1) blocks = 1;
+  k_fill_f32<<<(unsigned)blocks, 256, 0, st>>>(p, n, v);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rope_table(float2* tab, int n_pos, int half, double theta, cudaStream_t st) {
+  long long n = (long long)n_pos * half;
+  long long blocks = (n + 255) / 256;
+  if (blocks > 4096) blocks = 4096;
+  k_rope_table<<<(unsigned)blocks, 256, 0, st>>>(tab, n_pos, half, theta);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_embed(const void* E, bool is_bf16, const int* tok, float* x, int rows, int d, int V, int* err,
+                         cudaStream_t st) {
+  if (is_bf16)
+    return launch_pdl(k_embed<bf16>, dim3(rows), dim3(256), st, reinterpret_cast<const bf16*>(E), tok, x, d, V, err);
+  return launch_pdl(k_embed<float>, dim3(rows), dim3(256), st, reinterpret_cast<const float*>(E), tok, x, d, V, err);
+}
+
+cudaError_t launch_rmsnorm(const float* x, const float* gain, void* y, bool is_bf16, int rows, int d, float eps,
+                           cudaStream_t st) {
+  if (is_bf16)
+    return launch_pdl(k_rmsnorm<bf16>, dim3(rows), dim3(256), st, x, gain, reinterpret_cast<bf16*>(y), d, eps);
+  return launch_pdl(k_rmsnorm<float>, dim3(rows), dim3(256), st, x, gain, reinterpret_cast<float*>(y), d, eps);
+}
+
+}  // namespace jf

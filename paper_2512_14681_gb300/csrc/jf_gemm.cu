@@ -1,0 +1,483 @@
+// Weight-streaming projections of the forward pass (Eq. 3: one pass over all in-flight rows):
+// Y[m, n] = sum_k X[m, k] W[n, k] for the QKV, O, gate/up, down and LM-head matrices.
+//
+// bf16 path: tcgen05 tensor cores, "swap-AB" so that 128 weight rows form the MMA's M side and
+// the (few) in-flight tokens its N side; weights and activations arrive by TMA with 128-byte
+// swizzle into a multi-stage mbarrier pipeline; the fp32 accumulator lives in tensor memory.
+// fp32 path (small fp32 models): a SIMT mainloop with the same tile shape and epilogues.
+//
+// Split-K is deterministic: partial tiles go to a workspace and the last CTA of a tile (atomic
+// ticket, no waiting) adds them in split order. Every output element's reduction order is fixed
+// by the weight shape alone, so a row's result does not depend on how many rows are in flight.
+#include "jf_device.cuh"
+#include "jf_internal.h"
+
+namespace jf {
+namespace {
+
+constexpr int A_STAGE_BYTES = kTileN * kTileK * 2;  // 16 KB of weights per stage
+
+template <int BN>
+struct TcCfg {
+  static constexpr int B_STAGE_BYTES = BN * kTileK * 2;
+  static constexpr int STAGE_BYTES = A_STAGE_BYTES + B_STAGE_BYTES;
+  static constexpr int BUDGET = BN >= 160 ? 200 * 1024 : 104 * 1024;
+  static constexpr int S0 = BUDGET / STAGE_BYTES;
+  static constexpr int STAGES = S0 < 2 ? 2 : (S0 > 8 ? 8 : S0);
+  static constexpr int TMEM_COLS = BN <= 32 ? 32 : (BN <= 64 ? 64 : (BN <= 128 ? 128 : 256));
+  static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + 256;
+};
+
+JF_DEV uint8_t* align1024(uint8_t* p) {
+  return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
+}
+
+// ---------------------------------------------------------------------------------------------
+// Epilogue on one 16-column chunk: thread `row` (0..127) holds v[j] = Y[m0 + c0 + j, n0 + row].
+// xs: shared staging [16][128] fp32 (exchange between the two halves of a tile).
+// ---------------------------------------------------------------------------------------------
+template <typename T>
+JF_DEV void epilogue_chunk(const GemmEpi& e, const float (&v)[16], int row, int n0, int m0, int c0, float* xs,
+                           int n_tile, int n_tiles) {
+  const int n = n0 + row;
+  const int kind = e.kind;
+  if (kind == EPI_STORE || kind == EPI_RESID) {
+    if (n < e.N) {
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        const int m = m0 + c0 + j;
+        if (m < e.M) {
+          if (kind == EPI_STORE) e.y[(size_t)m * e.ldy + n] = v[j];
+          else e.x[(size_t)m * e.ldx + n] += v[j];
+        }
+      }
+    }
+    return;
+  }
+  if (kind == EPI_QKV || kind == EPI_SWIGLU) {
+#pragma unroll
+    for (int j = 0; j < 16; ++j) xs[j * 128 + row] = v[j];
+    __syncthreads();
+    if (kind == EPI_QKV) {
+      const int hd = e.head_dim, half = hd >> 1;
+      const int i = n % hd;
+      const bool is_q = n < e.n_q;
+      const bool is_k = !is_q && n < e.n_q + e.n_kv;
+      const bool rot = is_q || is_k;
+      const int partner = (i < half) ? row + half : row - half;
+      T* dst;
+      size_t stride;
+      if (is_q) { dst = reinterpret_cast<T*>(e.q_out) + n; stride = (size_t)e.n_q; }
+      else if (is_k) { dst = reinterpret_cast<T*>(e.k_out) + (n - e.n_q); stride = (size_t)e.n_kv; }
+      else { dst = reinterpret_cast<T*>(e.v_out) + (n - e.n_q - e.n_kv); stride = (size_t)e.n_kv; }
+      if (n < e.N) {
+#pragma unroll 4
+        for (int j = 0; j < 16; ++j) {
+          const int m = m0 + c0 + j;
+          if (m >= e.M) break;
+          float out = xs[j * 128 + row];
+          if (rot) {
+            const float2 cs = e.rope[(size_t)e.pos[m] * half + (i % half)];
+            const float x2 = xs[j * 128 + partner];
+            out = (i < half) ? (out * cs.x - x2 * cs.y) : (out * cs.x + x2 * cs.y);
+          }
+          dst[(size_t)m * stride] = to_act<T>(out);
+        }
+      }
+    } else {
+      if (row < 64) {
+        const int f = n_tile * 64 + row;
+#pragma unroll 4
+        for (int j = 0; j < 16; ++j) {
+          const int m = m0 + c0 + j;
+          if (m >= e.M) break;
+          const float g = xs[j * 128 + row], u = xs[j * 128 + row + 64];
+          reinterpret_cast<T*>(e.act)[(size_t)m * e.ld_act + f] = to_act<T>(silu_f(g) * u);
+        }
+      }
+    }
+    __syncthreads();
+    return;
+  }
+  // EPI_ARGMAX: best (value, index) and runner-up value over this tile's 128 vocabulary rows
+  {
+    float* red = xs;  // [4 warps][16 cols][3]
+    const int warp = row >> 5, lane = row & 31;
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      float b1 = (n < e.N) ? v[j] : -INFINITY;
+      int bi = (n < e.N) ? n : 0x7fffffff;
+      float b2 = -INFINITY;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const float o1 = __shfl_xor_sync(0xffffffffu, b1, o);
+        const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+        const float o2 = __shfl_xor_sync(0xffffffffu, b2, o);
+        if (better(o1, oi, b1, bi)) { b2 = fmaxf(b1, o2); b1 = o1; bi = oi; }
+        else { b2 = fmaxf(b2, o1); }
+      }
+      if (lane == 0) {
+        red[(warp * 16 + j) * 3 + 0] = b1;
+        red[(warp * 16 + j) * 3 + 1] = __int_as_float(bi);
+        red[(warp * 16 + j) * 3 + 2] = b2;
+      }
+    }
+    __syncthreads();
+    if (row < 16) {
+      const int j = row, m = m0 + c0 + j;
+      float b1 = red[j * 3 + 0], b2 = red[j * 3 + 2];
+      int bi = __float_as_int(red[j * 3 + 1]);
+      for (int w = 1; w < 4; ++w) {
+        const float o1 = red[(w * 16 + j) * 3 + 0], o2 = red[(w * 16 + j) * 3 + 2];
+        const int oi = __float_as_int(red[(w * 16 + j) * 3 + 1]);
+        if (better(o1, oi, b1, bi)) { b2 = fmaxf(b1, o2); b1 = o1; bi = oi; }
+        else { b2 = fmaxf(b2, o1); }
+      }
+      if (m < e.M) {
+        const size_t at = (size_t)m * n_tiles + n_tile;
+        e.am_v1[at] = b1;
+        e.am_i1[at] = bi;
+        e.am_v2[at] = b2;
+      }
+    }
+    __syncthreads();
+  }
+}
+
+// Last CTA of a token tile: reduce the per-tile argmax partials of rows m0..m0+BN-1.
+JF_DEV void argmax_finish(const GemmEpi& e, int m0, int BN, int n_tiles, int tid) {
+  const int warp = tid >> 5, lane = tid & 31;
+  for (int r = warp; r < BN; r += 4) {
+    const int m = m0 + r;
+    if (m >= e.M) break;
+    float b1 = -INFINITY, b2 = -INFINITY;
+    int bi = 0x7fffffff;
+    for (int t = lane; t < n_tiles; t += 32) {
+      const size_t at = (size_t)m * n_tiles + t;
+      const float o1 = __ldcg(e.am_v1 + at), o2 = __ldcg(e.am_v2 + at);
+      const int oi = __ldcg(e.am_i1 + at);
+      if (better(o1, oi, b1, bi)) { b2 = fmaxf(b1, o2); b1 = o1; bi = oi; }
+      else { b2 = fmaxf(b2, o1); }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float o1 = __shfl_xor_sync(0xffffffffu, b1, o);
+      const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+      const float o2 = __shfl_xor_sync(0xffffffffu, b2, o);
+      if (better(o1, oi, b1, bi)) { b2 = fmaxf(b1, o2); b1 = o1; bi = oi; }
+      else { b2 = fmaxf(b2, o1); }
+    }
+    if (lane == 0) {
+      e.am_out[m] = bi;
+      if (e.top2_out) { e.top2_out[2 * m] = b1; e.top2_out[2 * m + 1] = b2; }
+    }
+  }
+}
+
+// Shared tail of both mainloops: ticketing for split-K and argmax, then the epilogue.
+// get(c0, v) fills this thread's 16 accumulator values of columns c0..c0+15.
+template <typename T, int BN, typename Get>
+JF_DEV void finish_tile(const GemmParams& p, Get get, float* xs, int* sflag) {
+  const int tid = threadIdx.x;
+  const int n_tile = blockIdx.x, split = blockIdx.y, m_tile = blockIdx.z;
+  const int n0 = n_tile * kTileN, m0 = m_tile * BN;
+  const int tile_lin = m_tile * p.n_tiles + n_tile;
+  int ncols = p.M - m0;
+  if (ncols > BN) ncols = BN;
+  const int nchunks = (ncols + 15) >> 4;
+  if (p.k_splits == 1) {
+    for (int c = 0; c < nchunks; ++c) {
+      float v[16];
+      get(c * 16, v);
+      epilogue_chunk<T>(p.epi, v, tid, n0, m0, c * 16, xs, n_tile, p.n_tiles);
+    }
+  } else {
+    float* mine = p.ws + ((size_t)tile_lin * p.k_splits + split) * (size_t)BN * kTileN;
+    for (int c = 0; c < nchunks; ++c) {
+      float v[16];
+      get(c * 16, v);
+#pragma unroll
+      for (int j = 0; j < 16; ++j) mine[(c * 16 + j) * kTileN + tid] = v[j];
+    }
+    __threadfence();
+    __syncthreads();
+    if (tid == 0) {
+      const int t = atomicAdd(p.tile_counter + tile_lin, 1);
+      *sflag = (t == p.k_splits - 1);
+    }
+    __syncthreads();
+    if (!*sflag) return;
+    __threadfence();
+    const float* base = p.ws + (size_t)tile_lin * p.k_splits * (size_t)BN * kTileN;
+    for (int c = 0; c < nchunks; ++c) {
+      float v[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) v[j] = 0.0f;
+      for (int s = 0; s < p.k_splits; ++s) {
+        const float* src = base + (size_t)s * BN * kTileN;
+#pragma unroll
+        for (int j = 0; j < 16; ++j) v[j] += __ldcg(src + (c * 16 + j) * kTileN + tid);
+      }
+      epilogue_chunk<T>(p.epi, v, tid, n0, m0, c * 16, xs, n_tile, p.n_tiles);
+    }
+    if (tid == 0) p.tile_counter[tile_lin] = 0;
+  }
+  if (p.epi.kind == EPI_ARGMAX) {
+    __threadfence();
+    __syncthreads();
+    if (tid == 0) {
+      const int t = atomicAdd(p.epi.am_counter + m_tile, 1);
+      *sflag = (t == p.n_tiles - 1);
+    }
+    __syncthreads();
+    if (*sflag) {
+      __threadfence();
+      argmax_finish(p.epi, m0, BN, p.n_tiles, tid);
+      if (tid == 0) p.epi.am_counter[m_tile] = 0;
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------------------------
+// bf16 tcgen05 kernel. 128 threads: thread 0 = TMA producer, thread 32 = MMA issuer, then all
+// four warps drain the accumulator (warp w reads TMEM lanes 32w .. 32w+31).
+// ---------------------------------------------------------------------------------------------
+template <int BN>
+__global__ void __launch_bounds__(128, 1)
+    k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const GemmParams p) {
+  using Cfg = TcCfg<BN>;
+  constexpr int S = Cfg::STAGES;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + S * A_STAGE_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sB + S * Cfg::B_STAGE_BYTES);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * S + 1);
+  int* sflag = reinterpret_cast<int*>(tmem_slot + 1);
+  int* sok = sflag + 1;
+
+  const int tid = threadIdx.x, warp = tid >> 5;
+  const int split = blockIdx.y;
+  const int n0 = blockIdx.x * kTileN, m0 = blockIdx.z * BN;
+  const int kb_begin = (int)(((long long)p.kb_total * split) / p.k_splits);
+  const int kb_end = (int)(((long long)p.kb_total * (split + 1)) / p.k_splits);
+  const int nkb = kb_end - kb_begin;
+  const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + S), accum = smem_u32(bars + 2 * S);
+
+  if (warp == 0) {
+    tmem_alloc(smem_u32(tmem_slot), Cfg::TMEM_COLS);
+    tmem_relinquish();
+  }
+  if (tid == 32) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(full0 + 8 * s, 1);
+      mbar_init(empty0 + 8 * s, 1);
+    }
+    mbar_init(accum, 1);
+    *sok = 1;
+    fence_mbar_init();
+  }
+  if (tid == 64) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (tid == 0) {
+    // producer: weights do not depend on earlier kernels, so the first stages are requested
+    // before waiting for the previous kernel of the chain.
+    const uint64_t polA = l2_policy_evict_first(), polB = l2_policy_evict_last();
+    const int pre = nkb < S ? nkb : S;
+    for (int i = 0; i < pre; ++i) {
+      mbar_arrive_expect_tx(full0 + 8 * i, Cfg::STAGE_BYTES);
+      tma_load_2d(smem_u32(sA + i * A_STAGE_BYTES), &tmA, full0 + 8 * i, (kb_begin + i) * kTileK, n0, polA);
+    }
+    pdl_wait();
+    for (int i = 0; i < pre; ++i)
+      tma_load_2d(smem_u32(sB + i * Cfg::B_STAGE_BYTES), &tmB, full0 + 8 * i, (kb_begin + i) * kTileK, m0, polB);
+    for (int i = pre; i < nkb; ++i) {
+      const int s = i % S;
+      const uint32_t ph = (uint32_t)((i / S) - 1) & 1u;
+      if (!mbar_wait_bounded(empty0 + 8 * s, ph, JF_WAIT_LIMIT_NS)) {
+        jf_set_error(p.err, JF_DERR_TIMEOUT_MMA);
+        *sok = 0;
+        break;
+      }
+      mbar_arrive_expect_tx(full0 + 8 * s, Cfg::STAGE_BYTES);
+      tma_load_2d(smem_u32(sA + s * A_STAGE_BYTES), &tmA, full0 + 8 * s, (kb_begin + i) * kTileK, n0, polA);
+      tma_load_2d(smem_u32(sB + s * Cfg::B_STAGE_BYTES), &tmB, full0 + 8 * s, (kb_begin + i) * kTileK, m0, polB);
+    }
+  } else if (tid == 32) {
+    pdl_wait();
+    constexpr uint32_t idesc = idesc_bf16_f32(kTileN, BN);
+    for (int i = 0; i < nkb; ++i) {
+      const int s = i % S;
+      if (!mbar_wait_bounded(full0 + 8 * s, (uint32_t)(i / S) & 1u, JF_WAIT_LIMIT_NS)) {
+        jf_set_error(p.err, JF_DERR_TIMEOUT_TMA);
+        *sok = 0;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t a = smem_u32(sA + s * A_STAGE_BYTES), b = smem_u32(sB + s * Cfg::B_STAGE_BYTES);
+#pragma unroll
+      for (int kk = 0; kk < kTileK / 16; ++kk)
+        tc_mma_bf16(tmem, sdesc_k_sw128(a + kk * 32), sdesc_k_sw128(b + kk * 32), idesc, (i | kk) != 0);
+      tc_commit(empty0 + 8 * s);
+    }
+    tc_commit(accum);
+  } else {
+    pdl_wait();
+  }
+  __syncwarp();
+  const bool acc_ok = mbar_wait_bounded(accum, 0, JF_WAIT_LIMIT_NS);
+  tc_fence_after();
+  if (!acc_ok) jf_set_error(p.err, JF_DERR_TIMEOUT_EPI);
+  __syncthreads();
+  pdl_launch_dependents();
+  if (acc_ok && *sok) {
+    float* xs = reinterpret_cast<float*>(sA);
+    const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+    auto get = [&](int c0, float (&v)[16]) { tmem_ld16(tmem + lane_base + (uint32_t)c0, v); };
+    finish_tile<bf16, BN>(p, get, xs, sflag);
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tmem, Cfg::TMEM_COLS);
+}
+
+// ---------------------------------------------------------------------------------------------
+// fp32 SIMT kernel: thread `row` accumulates Y[m0 .. m0+31, n0 + row] over K in fp32, in
+// increasing k, with the token tile staged in shared memory.
+// ---------------------------------------------------------------------------------------------
+constexpr int F32_BN = 32;
+constexpr int F32_BK = 32;
+
+__global__ void __launch_bounds__(128) k_gemm_f32(const float* __restrict__ W, const float* __restrict__ X,
+                                                  const GemmParams p) {
+  __shared__ float xt[F32_BN][F32_BK + 1];
+  __shared__ float xs[16 * 128];
+  __shared__ int sflag;
+  const int tid = threadIdx.x;
+  const int n0 = blockIdx.x * kTileN, m0 = blockIdx.z * F32_BN;
+  const int n = n0 + tid;
+  pdl_wait();
+  float acc[F32_BN];
+#pragma unroll
+  for (int j = 0; j < F32_BN; ++j) acc[j] = 0.0f;
+  for (int k0 = 0; k0 < p.K; k0 += F32_BK) {
+    for (int i = tid; i < F32_BN * F32_BK; i += 128) {
+      const int r = i / F32_BK, c = i % F32_BK;
+      const int m = m0 + r, k = k0 + c;
+      xt[r][c] = (m < p.M && k < p.K) ? X[(size_t)m * p.K + k] : 0.0f;
+    }
+    __syncthreads();
+    if (n < p.N) {
+      const float* wr = W + (size_t)n * p.K + k0;
+      const int kmax = (p.K - k0) < F32_BK ? (p.K - k0) : F32_BK;
+      for (int c = 0; c < kmax; ++c) {
+        const float w = wr[c];
+#pragma unroll
+        for (int j = 0; j < F32_BN; ++j) acc[j] = fmaf(w, xt[j][c], acc[j]);
+      }
+    }
+    __syncthreads();
+  }
+  pdl_launch_dependents();
+  auto get = [&](int c0, float (&v)[16]) {
+#pragma unroll
+    for (int j = 0; j < 16; ++j) v[j] = 0.0f;
+#pragma unroll
+    for (int cc = 0; cc < F32_BN; cc += 16)
+      if (cc == c0) {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) v[j] = acc[cc + j];
+      }
+  };
+  finish_tile<float, F32_BN>(p, get, xs, &sflag);
+}
+
+template <int BN>
+cudaError_t launch_tc(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmParams& p, cudaStream_t st) {
+  using Cfg = TcCfg<BN>;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.n_tiles, p.k_splits, p.m_tiles);
+  cfg.blockDim = dim3(128);
+  cfg.dynamicSmemBytes = Cfg::SMEM;
+  cfg.stream = st;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, k_gemm_tc<BN>, tmA, tmB, p);
+}
+
+template <int BN>
+cudaError_t prep_tc() {
+  return cudaFuncSetAttribute(k_gemm_tc<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<BN>::SMEM);
+}
+
+}  // namespace
+
+// Opt the tcgen05 kernels into their dynamic shared-memory sizes (once per process, outside any
+// stream capture).
+cudaError_t gemm_prepare() {
+  cudaError_t e;
+  if ((e = prep_tc<16>()) != cudaSuccess) return e;
+  if ((e = prep_tc<32>()) != cudaSuccess) return e;
+  if ((e = prep_tc<64>()) != cudaSuccess) return e;
+  if ((e = prep_tc<128>()) != cudaSuccess) return e;
+  if ((e = prep_tc<160>()) != cudaSuccess) return e;
+  return prep_tc<256>();
+}
+
+int gemm_bn_for(int M) {
+  if (M <= 16) return 16;
+  if (M <= 32) return 32;
+  if (M <= 64) return 64;
+  if (M <= 128) return 128;
+  if (M <= 160) return 160;
+  return 256;
+}
+
+size_t gemm_smem_bytes(int bn) {
+  switch (bn) {
+    case 16: return TcCfg<16>::SMEM;
+    case 32: return TcCfg<32>::SMEM;
+    case 64: return TcCfg<64>::SMEM;
+    case 128: return TcCfg<128>::SMEM;
+    case 160: return TcCfg<160>::SMEM;
+    default: return TcCfg<256>::SMEM;
+  }
+}
+
+cudaError_t launch_gemm_bf16(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmParams& p, int bn,
+                             cudaStream_t st) {
+  switch (bn) {
+    case 16: return launch_tc<16>(tmA, tmB, p, st);
+    case 32: return launch_tc<32>(tmA, tmB, p, st);
+    case 64: return launch_tc<64>(tmA, tmB, p, st);
+    case 128: return launch_tc<128>(tmA, tmB, p, st);
+    case 160: return launch_tc<160>(tmA, tmB, p, st);
+    case 256: return launch_tc<256>(tmA, tmB, p, st);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+cudaError_t launch_gemm_f32(const float* W, const float* X, const GemmParams& p, cudaStream_t st) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.n_tiles, 1, p.m_tiles);
+  cfg.blockDim = dim3(128);
+  cfg.stream = st;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, k_gemm_f32, W, X, p);
+}
+
+}  // namespace jf

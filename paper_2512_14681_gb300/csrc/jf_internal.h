@@ -1,0 +1,114 @@
+// Internal structures shared by the libjf host runtime and its kernels (not part of the C ABI).
+#pragma once
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace jf {
+
+// Device error codes written into the context's error word (first writer wins).
+enum DeviceError : int {
+  JF_DERR_NONE = 0,
+  JF_DERR_TIMEOUT_TMA = 1,   // a TMA transfer never completed its mbarrier
+  JF_DERR_TIMEOUT_MMA = 2,   // an MMA commit never arrived
+  JF_DERR_TIMEOUT_EPI = 3,   // the accumulator barrier never completed
+  JF_DERR_BOUNDS = 4,        // a page-table / token / position index was out of range
+  JF_DERR_STATE = 5,         // inconsistent decode state detected on the device
+};
+
+
+constexpr int kPage = 16;         // tokens per KV page
+constexpr int kTileN = 128;       // weight rows per GEMM tile (tcgen05 M)
+constexpr int kTileK = 64;        // K elements per GEMM pipeline stage
+constexpr int kAttnChunk = 128;   // keys per split-KV chunk, aligned to absolute positions
+constexpr int kAttnQRows = 64;    // (token, head) query rows per attention work unit
+constexpr int kMaxSeqs = 64;
+constexpr int kMaxChains = 256;
+
+// A chain: in-flight rows row0 .. row0+nrows-1 of sequence `seq` at consecutive positions
+// pos0 .. pos0+nrows-1, where pos0 equals the sequence's committed length. Each row attends to
+// the whole committed cache and to the rows of its own chain at positions <= its own.
+struct Chain {
+  int seq, row0, nrows, pos0;
+};
+
+// Attention work decomposition computed on the device once per forward.
+struct AttnUnit {
+  int chain, kvh, qt, n_chunks, slot0;
+};
+struct AttnPlan {
+  int n_units, n_items, n_slots, pad;
+};
+
+enum EpiKind : int { EPI_STORE = 0, EPI_RESID = 1, EPI_QKV = 2, EPI_SWIGLU = 3, EPI_ARGMAX = 4 };
+
+struct GemmEpi {
+  int kind;
+  int M, N;
+  // EPI_STORE: y[m * ldy + n] = v (fp32)
+  float* y;
+  int ldy;
+  // EPI_RESID: x[m * ldx + n] += v (fp32 residual stream)
+  float* x;
+  int ldx;
+  // EPI_QKV: rotary embedding on q/k features, then q -> q_out[m][Hq][hd], k/v -> k_out/v_out[m][Hkv][hd]
+  void* q_out;
+  void* k_out;
+  void* v_out;
+  int n_q, n_kv, head_dim;
+  const int* pos;
+  const float2* rope;   // [max_pos][hd/2] (cos, sin)
+  // EPI_SWIGLU: tile t holds gate rows 64t..64t+63 then the matching up rows; act[m][64t + i]
+  void* act;
+  int ld_act;
+  // EPI_ARGMAX: per (row, tile) partial (v1, i1, v2), ticket per token tile, final argmax/top2
+  float* am_v1;
+  int* am_i1;
+  float* am_v2;
+  int* am_counter;
+  int* am_out;
+  float* top2_out;
+};
+
+struct GemmParams {
+  int N, K, M;
+  int n_tiles, m_tiles, k_splits, kb_total;
+  float* ws;           // split-K partials [m_tiles*n_tiles][k_splits][BN][128]
+  int* tile_counter;   // [m_tiles*n_tiles], zero between launches
+  int* err;
+  GemmEpi epi;
+};
+
+struct AttnParams {
+  const void* q;        // [R][Hq][hd]
+  const void* k_inf;    // this layer's in-flight K [R][Hkv][hd]
+  const void* v_inf;
+  const void* k_pages;  // this layer's K pages [n_pages][Hkv][16][hd]
+  const void* v_pages;
+  const int* page_table;  // [max_seqs][pages_per_seq]
+  int pages_per_seq;
+  int n_pages;
+  const int* seq_len;   // committed length per sequence
+  const Chain* chains;
+  const int* n_chains_dev;
+  const AttnPlan* plan;
+  const AttnUnit* units;
+  const int2* items;    // (unit, chunk)
+  float* ws_o;          // [slot][64][hd]
+  float* ws_ml;         // [slot][64][2]
+  int* unit_counter;    // [max_units]
+  void* out;            // [R][Hq*hd]
+  int Hq, Hkv, hd;
+  float scale_log2;     // log2(e) / sqrt(hd)
+  int* err;
+};
+
+// Host-side launch helpers (jf_kernels.cu). All launches use programmatic dependent launch.
+cudaError_t launch_gemm_bf16(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmParams& p, int bn,
+                             cudaStream_t st);
+cudaError_t launch_gemm_f32(const float* W, const float* X, const GemmParams& p, cudaStream_t st);
+int gemm_bn_for(int M);
+size_t gemm_smem_bytes(int bn);
+
+}  // namespace jf

@@ -1,0 +1,228 @@
+"""Python face of libjf: a Context owning a device arena (PyTorch memory) and a CUDA stream.
+
+Every method marshals arguments and calls one C entry point of include/jf.h; the Jacobi
+iteration itself (forward pass, greedy argmax, acceptance, KV commit, draft bookkeeping) runs in
+libjf's CUDA kernels.
+"""
+from __future__ import annotations
+
+import ctypes as C
+from dataclasses import dataclass
+
+import numpy as np
+
+from . import _lib as J
+from .inputs import ModelShape
+
+
+def _check(lib, ctx, status: int):
+    if status != J.JF_OK:
+        msg = lib.jf_last_error(ctx).decode() if ctx else ""
+        raise J.JfError(status, msg)
+
+
+def _i32p(a):
+    return a.ctypes.data_as(C.POINTER(C.c_int32))
+
+
+@dataclass
+class Gen:
+    """Generation parameters (see jf_gen_params in include/jf.h)."""
+    block_size: int = 8
+    n_blocks: int = 1
+    spawn_ratio: float = 0.0
+    pool_size: int = 0
+    ngram_len: int = 0
+    cand_per_iter: int = 0
+    mode: str = "block"
+    init: str = "repeat"
+    inject_p: float = 0.0
+    seed: int = 0
+    max_new: int = 64
+    eos_id: int = -1
+
+    def c_struct(self, truth_ptr=None, truth_len=0) -> J.GenParams:
+        mode = {"block": J.JF_MODE_BLOCK, "window": J.JF_MODE_WINDOW, "ar": J.JF_MODE_AR}[self.mode]
+        init = {"repeat": J.JF_INIT_REPEAT, "inject": J.JF_INIT_INJECT}[self.init]
+        return J.GenParams(self.block_size, self.n_blocks, self.spawn_ratio, self.pool_size, self.ngram_len,
+                           self.cand_per_iter, mode, init, self.inject_p, self.seed, self.max_new, self.eos_id,
+                           truth_ptr, truth_len)
+
+
+@dataclass
+class GenOut:
+    tokens: np.ndarray      # [n_seqs, max_new]
+    counts: np.ndarray      # [iterations, n_seqs] tokens committed per iteration (-1 = inactive)
+    rows: np.ndarray        # [iterations] in-flight rows per iteration
+    iterations: int
+    prefill_ms: float
+    decode_ms: float
+    kernel_launches: int = 0
+
+
+def model_config(shape: ModelShape) -> J.ModelConfig:
+    return J.ModelConfig(shape.n_layers, shape.d_model, shape.n_heads, shape.n_kv_heads, shape.head_dim,
+                         shape.d_ff, shape.vocab, shape.rms_eps, shape.rope_theta,
+                         J.JF_BF16 if shape.bf16 else J.JF_F32)
+
+
+class Context:
+    """A libjf context on the current CUDA device."""
+
+    def __init__(self, shape: ModelShape, max_seqs: int = 1, max_ctx: int = 2048, max_rows: int = 64,
+                 logits_rows: int = 0, stream=None):
+        import torch
+
+        self.lib = J.load()
+        self.shape = shape
+        self.mc = model_config(shape)
+        self.torch = torch
+        self.stream = stream if stream is not None else torch.cuda.Stream()
+        rc = J.RuntimeConfig(max_seqs, max_ctx, max_rows, logits_rows, None, 0, self.stream.cuda_stream)
+        nbytes = C.c_size_t()
+        _check(self.lib, None, self.lib.jf_arena_bytes(C.byref(self.mc), C.byref(rc), C.byref(nbytes)))
+        self.arena = torch.empty(nbytes.value, dtype=torch.uint8, device="cuda")
+        rc.device_arena = self.arena.data_ptr()
+        rc.arena_bytes = nbytes.value
+        self.rc = rc
+        h = C.c_void_p()
+        torch.cuda.synchronize()
+        _check(self.lib, None, self.lib.jf_create(C.byref(self.mc), C.byref(rc), C.byref(h)))
+        self.h = h
+        self.max_rows = max_rows
+        self.max_ctx = max_ctx
+
+    def close(self):
+        if getattr(self, "h", None):
+            self.lib.jf_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def _c(self, status):
+        _check(self.lib, self.h, status)
+
+    # -- weights -----------------------------------------------------------------------
+    def init_random_weights(self, seed: int = 0, std: float = 0.02):
+        self._c(self.lib.jf_init_random_weights(self.h, seed, std))
+
+    def save_weights(self, path: str):
+        self._c(self.lib.jf_save_weights(self.h, path.encode()))
+
+    def load_weights(self, path: str):
+        self._c(self.lib.jf_load_weights(self.h, path.encode()))
+
+    def get_weights(self, tensor_id: int, start: int, count: int) -> np.ndarray:
+        out = np.empty(count, dtype=np.float32)
+        self._c(self.lib.jf_get_weights(self.h, tensor_id, start, count,
+                                        out.ctypes.data_as(C.POINTER(C.c_float))))
+        return out
+
+    # -- sequences ---------------------------------------------------------------------
+    def prefill(self, seq: int, prompt) -> int:
+        p = np.ascontiguousarray(prompt, dtype=np.int32)
+        nt = C.c_int32()
+        self._c(self.lib.jf_prefill(self.h, seq, _i32p(p), p.size, C.byref(nt)))
+        return int(nt.value)
+
+    def truncate(self, seq: int, length: int):
+        self._c(self.lib.jf_truncate(self.h, seq, length))
+
+    def seq_len(self, seq: int) -> int:
+        v = C.c_int()
+        self._c(self.lib.jf_seq_len(self.h, seq, C.byref(v)))
+        return int(v.value)
+
+    def jacobi_step(self, seq: int, blocks, draft):
+        """blocks: list of (kind, start_pos, len, parent). Returns dict of outputs."""
+        bl = (J.Block * len(blocks))(*[J.Block(*b) for b in blocks])
+        d = np.ascontiguousarray(draft, dtype=np.int32)
+        counts = np.zeros(len(blocks), dtype=np.int32)
+        committed = np.zeros(max(b[2] for b in blocks), dtype=np.int32)
+        n_comm = C.c_int32()
+        pred = np.zeros(d.size, dtype=np.int32)
+        top2 = np.zeros((d.size, 2), dtype=np.float32)
+        self._c(self.lib.jf_jacobi_step(self.h, seq, len(blocks), bl, _i32p(d), _i32p(counts), _i32p(committed),
+                                        C.byref(n_comm), _i32p(pred), top2.ctypes.data_as(C.POINTER(C.c_float))))
+        return dict(counts=counts, committed=committed[: n_comm.value], predictions=pred, top2=top2)
+
+    def forward_logits(self, seq: int, tokens, want_logits=True, want_hidden=True):
+        t = np.ascontiguousarray(tokens, dtype=np.int32)
+        n = t.size
+        logits = np.empty((n, self.shape.vocab), dtype=np.float32) if want_logits else None
+        hidden = np.empty((n, self.shape.d_model), dtype=np.float32) if want_hidden else None
+        am = np.empty(n, dtype=np.int32)
+        fp = C.POINTER(C.c_float)
+        self._c(self.lib.jf_forward_logits(self.h, seq, n, _i32p(t),
+                                           logits.ctypes.data_as(fp) if logits is not None else None,
+                                           hidden.ctypes.data_as(fp) if hidden is not None else None, _i32p(am)))
+        return logits, hidden, am
+
+    # -- generation --------------------------------------------------------------------
+    def generate(self, prompts, gen: Gen, truth=None, log_cap: int = 4096) -> GenOut:
+        """Host buffers in and out (jf_generate)."""
+        ps = [np.ascontiguousarray(p, dtype=np.int32) for p in prompts]
+        n = len(ps)
+        arr = (C.POINTER(C.c_int32) * n)(*[_i32p(p) for p in ps])
+        lens = np.array([p.size for p in ps], dtype=np.int32)
+        tr = None
+        tlen = 0
+        if truth is not None:
+            tr = np.ascontiguousarray(truth, dtype=np.int32)
+            tlen = tr.shape[-1]
+        gp = gen.c_struct(tr.ctypes.data if tr is not None else None, tlen)
+        out = np.empty((n, gen.max_new), dtype=np.int32)
+        acc = np.full((log_cap, n), -1, dtype=np.int32)
+        rows = np.zeros(log_cap, dtype=np.int32)
+        st = J.GenStats(0, _i32p(acc), _i32p(rows), log_cap, 0.0, 0.0, 0)
+        self._c(self.lib.jf_generate(self.h, n, arr, _i32p(lens), C.byref(gp), _i32p(out), C.byref(st)))
+        it = st.iterations
+        return GenOut(out, acc[: min(it, log_cap)], rows[: min(it, log_cap)], it, st.prefill_ms, st.decode_ms,
+                      st.kernel_launches)
+
+    def generate_device(self, d_prompts, prompt_lens, gen: Gen, d_out, d_truth=None, truth_len=0,
+                        log_cap: int = 0):
+        """Device buffers (torch int32 CUDA tensors) in and out (jf_generate_device)."""
+        lens = np.ascontiguousarray(prompt_lens, dtype=np.int32)
+        gp = gen.c_struct(d_truth.data_ptr() if d_truth is not None else None, truth_len)
+        n = lens.size
+        acc = np.full((max(log_cap, 1), n), -1, dtype=np.int32)
+        rows = np.zeros(max(log_cap, 1), dtype=np.int32)
+        st = J.GenStats(0, _i32p(acc), _i32p(rows), log_cap, 0.0, 0.0, 0)
+        self._c(self.lib.jf_generate_device(self.h, n, d_prompts.data_ptr(), _i32p(lens), C.byref(gp),
+                                            d_out.data_ptr(), C.byref(st)))
+        it = st.iterations
+        return GenOut(None, acc[: min(it, log_cap)], rows[: min(it, log_cap)], it, st.prefill_ms, st.decode_ms,
+                      st.kernel_launches)
+
+    def set_profiling(self, on: bool):
+        self._c(self.lib.jf_set_profiling(self.h, 1 if on else 0))
+
+    def kernel_time(self, cls: int):
+        ms = C.c_double()
+        n = C.c_longlong()
+        self._c(self.lib.jf_kernel_time(self.h, cls, C.byref(ms), C.byref(n)))
+        return ms.value, n.value
+
+
+def op_gemm(W, X, k_splits: int = 0, stream=None):
+    """Y = X W^T through jf_op_gemm (torch CUDA tensors W [N,K], X [M,K], bf16 or fp32)."""
+    import torch
+
+    lib = J.load()
+    N, K = W.shape
+    M = X.shape[0]
+    dtype = J.JF_BF16 if W.dtype == torch.bfloat16 else J.JF_F32
+    nb = C.c_size_t()
+    _check(lib, None, lib.jf_op_gemm_workspace_bytes(N, K, M, k_splits, C.byref(nb)))
+    ws = torch.zeros(max(nb.value, 16), dtype=torch.uint8, device=W.device)
+    err = torch.zeros(1, dtype=torch.int32, device=W.device)
+    Y = torch.empty((M, N), dtype=torch.float32, device=W.device)
+    s = stream if stream is not None else torch.cuda.current_stream()
+    _check(lib, None, lib.jf_op_gemm(dtype, W.data_ptr(), X.data_ptr(), Y.data_ptr(), N, K, M, k_splits,
+                                     ws.data_ptr(), nb.value, err.data_ptr(), s.cuda_stream))
+    return Y, err, ws

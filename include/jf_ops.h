@@ -33,6 +33,25 @@ jf_status jf_op_gemm_workspace_bytes(int N, int K, int M, int k_splits, size_t* 
 jf_status jf_op_gemm(int dtype, const void* W, const void* X, float* Y, int N, int K, int M, int k_splits,
                      void* workspace, size_t workspace_bytes, int* err_word, void* cuda_stream);
 
+/* Size of the fixed device scratch of jf_op_gemm_noalloc (8 MiB). */
+#define JF_OP_GEMM_NOALLOC_SCRATCH_BYTES (8u << 20)
+
+/* jf_op_gemm without a workspace, for callers that cannot allocate device memory: code running
+ * inside a device-memory allocator's own hooks, or a process whose device memory is entirely
+ * reserved by another pool, cannot obtain the workspace jf_op_gemm asks for. (The paper has no
+ * counterpart; this is a library facility.)
+ * dtype is bf16 only: W [N][K], X [M][K] bf16 (device, 16-byte aligned, K % 8 == 0), Y fp32 [M][N].
+ * The split-K scratch is one static device array of JF_OP_GEMM_NOALLOC_SCRATCH_BYTES that every GPU
+ * loading libjf holds until the process exits; a shape whose jf_op_gemm_workspace_bytes() exceeds
+ * it is refused with JF_ECAPACITY before any launch. The call allocates nothing (no cudaMalloc,
+ * no cudaFree, no allocating library routine). Its first call on a device looks up the array's
+ * device address (cudaGetSymbolAddress) and sets kernel attributes, so make that first call before
+ * any stream capture. All calls share the array: calls that may overlap on the GPU (other streams,
+ * other threads) race on it and must be serialised by the caller; each call re-zeroes the tickets
+ * it uses before its kernel runs. err_word and cuda_stream as in jf_op_gemm. */
+jf_status jf_op_gemm_noalloc(const void* W, const void* X, float* Y, int N, int K, int M, int k_splits,
+                             int* err_word, void* cuda_stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -17,7 +17,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 OUT = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT, "libjf.so")
-SOURCES = ["jf_gemm.cu", "jf_attention.cu", "jf_elementwise.cu", "jf_decode.cu", "jf_runtime.cu"]
+SOURCES = ["jf_gemm.cu", "jf_attention.cu", "jf_elementwise.cu", "jf_decode.cu", "jf_runtime.cu", "jf_noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

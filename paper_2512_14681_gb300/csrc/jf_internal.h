@@ -110,5 +110,7 @@ cudaError_t launch_gemm_bf16(const CUtensorMap& tmA, const CUtensorMap& tmB, con
 cudaError_t launch_gemm_f32(const float* W, const float* X, const GemmParams& p, cudaStream_t st);
 int gemm_bn_for(int M);
 size_t gemm_smem_bytes(int bn);
+int gemm_default_splits(int n_tiles, int kb_total);
+bool encode_tmap_bf16(CUtensorMap* tm, const void* ptr, long long K, long long rows, int box_rows);
 
 }  // namespace jf

@@ -249,6 +249,12 @@ struct GraphRec {
 
 }  // namespace
 
+// Shared with the allocation-free GEMM entry point (jf_noalloc.cu).
+int jf::gemm_default_splits(int n_tiles, int kb_total) { return splits_for(n_tiles, kb_total); }
+bool jf::encode_tmap_bf16(CUtensorMap* tm, const void* ptr, long long K, long long rows, int box_rows) {
+  return make_tmap(tm, ptr, K, rows, box_rows);
+}
+
 struct jf_ctx {
   jf_model_config mc;
   jf_runtime_config rc;

@@ -226,3 +226,19 @@ def op_gemm(W, X, k_splits: int = 0, stream=None):
     _check(lib, None, lib.jf_op_gemm(dtype, W.data_ptr(), X.data_ptr(), Y.data_ptr(), N, K, M, k_splits,
                                      ws.data_ptr(), nb.value, err.data_ptr(), s.cuda_stream))
     return Y, err, ws
+
+
+def op_gemm_noalloc(W, X, k_splits: int = 0, stream=None):
+    """Y = X W^T through jf_op_gemm_noalloc: bf16 only, no workspace argument (the library's fixed
+    device scratch serves the split-K partials). Returns (Y, err_word, status)."""
+    import torch
+
+    lib = J.load()
+    N, K = W.shape
+    M = X.shape[0]
+    err = torch.zeros(1, dtype=torch.int32, device=W.device)
+    Y = torch.empty((M, N), dtype=torch.float32, device=W.device)
+    s = stream if stream is not None else torch.cuda.current_stream()
+    status = lib.jf_op_gemm_noalloc(W.data_ptr(), X.data_ptr(), Y.data_ptr(), N, K, M, k_splits, err.data_ptr(),
+                                    s.cuda_stream)
+    return Y, err, status

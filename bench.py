@@ -166,6 +166,11 @@ def run_gpu(args, rank, world, local_rank):
 
         dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
     shape = I.QWEN7B_BF16
+    if args.layers != shape.n_layers:
+        # reduced-depth copy of the 7B shape: small profiling case only, never a headline number
+        import dataclasses
+
+        shape = dataclasses.replace(shape, n_layers=args.layers, name=f"{shape.name}-{args.layers}layers")
     truth_len = NEW + 2 * BLOCK + 1
     # max_rows 512: the 1024-token prompt is prefilled in two 512-row forwards
     ctx = Context(shape, max_seqs=1, max_ctx=2048, max_rows=512)
@@ -240,6 +245,10 @@ def run_gpu(args, rank, world, local_rank):
     torch.cuda.synchronize()
     gu_ms, gu_n = ctx.kernel_time(0)
     at_ms, at_n = ctx.kernel_time(1)
+    class_names = ["gate_up", "attention", "all_gemms", "qkv", "o_proj", "down", "lm_head", "attn_combine", "rmsnorm",
+                   "other"]
+    prof = {nm: ctx.kernel_time(i) for i, nm in enumerate(class_names)}
+    prof_iters = max(1, prof["lm_head"][1])
     ctx.set_profiling(False)
 
     if rank != 0:
@@ -266,7 +275,8 @@ def run_gpu(args, rank, world, local_rank):
         "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic: uniform-random prompt, N(0,0.02) random weights, drafts injected from the model's own "
                 "greedy continuation",
-        "config": {"workload": WORKLOAD, "prompt": PROMPT_LEN, "block_size": BLOCK, "new_tokens": NEW,
+        "config": {"workload": WORKLOAD if args.layers == 28 else f"{WORKLOAD} ({args.layers}-layer profiling case)",
+                   "layers": shape.n_layers, "prompt": PROMPT_LEN, "block_size": BLOCK, "new_tokens": NEW,
                    "inject_p": P_INJECT, "kv_page_tokens": 16, "batch": 1,
                    "parallelism": "replicas" if world > 1 else "single-gpu",
                    "l2": "no flush: every step streams 14.1 GB of weights through the 129 MB L2"},
@@ -282,6 +292,7 @@ def run_gpu(args, rank, world, local_rank):
                      "bytes_per_launch": gu_bytes, "launches_timed": gu_n, "avg_launch_us": gu_avg_s * 1e6,
                      "peak_kind": peak_kind, "timing": "CUDA events around each launch in a profiled pass of the step"},
         "attention": {"launches_timed": at_n, "avg_launch_us": (at_ms / max(at_n, 1)) * 1000.0},
+        "profiled_breakdown_us_per_iteration": {nm: 1000.0 * ms / prof_iters for nm, (ms, n) in prof.items()},
         "clocks": clocks,
     }
     if args.cpu_baseline and world == 1:
@@ -302,6 +313,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
     ap.add_argument("--cpu-baseline-iters", type=int, default=2)
+    ap.add_argument("--layers", type=int, default=28, help="decoder layers (28 = the workload; fewer = profiling case)")
     args = ap.parse_args()
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))

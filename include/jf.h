@@ -181,9 +181,12 @@ jf_status jf_generate_device(jf_ctx* ctx, int n_seqs, const int32_t* d_prompts, 
                              const jf_gen_params* params, int32_t* d_out_tokens, jf_gen_stats* stats);
 
 /* Cumulative device time (ms, CUDA events) and launch count of one kernel class inside
- * jf_generate* decode iterations, when profiling is enabled with jf_set_profiling(ctx, 1).
- * kernel_class: 0 = gate/up projection GEMM (the largest weight stream), 1 = attention,
- * 2 = all projection GEMMs. */
+ * jf_generate* decode iterations, when profiling is enabled with jf_set_profiling(ctx, 1) (event
+ * records are then placed around every kernel of the iteration graph, which serialises them).
+ * kernel_class: 0 = gate/up projection (the largest weight stream), 1 = split-KV attention,
+ * 2 = all projection GEMMs, 3 = QKV projection, 4 = O projection, 5 = down projection,
+ * 6 = LM head + argmax, 7 = attention combine, 8 = RMSNorm, 9 = other (embedding, attention plan,
+ * acceptance, KV commit). jf_set_profiling resets the counters. */
 jf_status jf_set_profiling(jf_ctx* ctx, int enable);
 jf_status jf_kernel_time(jf_ctx* ctx, int kernel_class, double* total_ms, long long* launches);
 

@@ -65,27 +65,36 @@ JF_DEV uint32_t pack_bf16(float lo, float hi) {
 }
 
 // Address of the K (or V) row for absolute key position kp of unit (chain, kvh); null if the
-// position holds no key for this chain.
+// position holds no key for this chain. spage: the chunk's page ids (kp0 / 16 ...), resolved once.
 JF_DEV const bf16* key_row(const AttnParams& a, const bf16* pages, const bf16* inf, const Chain& ch, int kvh, int kp,
-                           int max_kp) {
+                           int max_kp, int kp0, const int* spage) {
   if (kp > max_kp) return nullptr;
   if (kp < ch.pos0) {
-    const int page = a.page_table[(size_t)ch.seq * a.pages_per_seq + (kp >> 4)];
+    const int page = spage[(kp - kp0) >> 4];
     if (page < 0 || page >= a.n_pages) return nullptr;
     return pages + (((size_t)page * a.Hkv + kvh) * kPage + (kp & 15)) * HD;
   }
   return inf + ((size_t)(ch.row0 + kp - ch.pos0) * a.Hkv + kvh) * HD;
 }
 
-__global__ void __launch_bounds__(128) k_attn_bf16(const AttnParams a) {
+// One work item = (unit, 128-key chunk). 8 warps: warp w computes query-row group w & 3 (16 rows)
+// against key sub-block w >> 2 (64 keys); the two sub-block partials of a row are merged in shared
+// memory, sub-block 0 first, so the chunk's arithmetic is fixed by absolute key positions.
+constexpr int ATT_THREADS = 256;
+
+__global__ void __launch_bounds__(ATT_THREADS, 1) k_attn_bf16(const AttnParams a) {
   extern __shared__ __align__(128) uint8_t sm[];
   uint8_t* sQ = sm;                       // 64 x 256 B
   uint8_t* sK = sm + TILE_BYTES;          // NSUB x 16 KB
   uint8_t* sV = sK + NSUB * TILE_BYTES;   // NSUB x 16 KB
-  __shared__ int s_last;
+  float* sO1 = reinterpret_cast<float*>(sK + TILE_BYTES);  // sub-block 1 partial O [64][128], reuses K1/V1
   __shared__ int s_rowpos[kAttnQRows];
+  __shared__ int s_page[kAttnChunk / kPage];
+  __shared__ float s_m1[kAttnQRows], s_l1[kAttnQRows];
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int rg = warp & 3, sb = warp >> 2;
+  pdl_launch_dependents();  // the next kernel may launch now
   pdl_wait();
   const int n_items = a.plan->n_items;
   const int G = a.Hq / a.Hkv;
@@ -108,8 +117,13 @@ __global__ void __launch_bounds__(128) k_attn_bf16(const AttnParams a) {
     const int max_kp = ch.pos0 + (qr0 + qrows - 1) / G;
     const int kp0 = chunk * kAttnChunk;
 
-    // stage Q (64 rows, zero beyond qrows) and the chunk's keys/values
-    for (int i = tid; i < kAttnQRows * 16; i += 128) {
+    if (tid < kAttnQRows) s_rowpos[tid] = (tid < qrows) ? ch.pos0 + (qr0 + tid) / G : -1;
+    if (tid < kAttnChunk / kPage) {
+      const int kp = kp0 + tid * kPage;
+      s_page[tid] = (kp < ch.pos0) ? a.page_table[(size_t)ch.seq * a.pages_per_seq + (kp >> 4)] : -1;
+    }
+    // stage Q (64 rows, zero beyond qrows)
+    for (int i = tid; i < kAttnQRows * 16; i += ATT_THREADS) {
       const int r = i >> 4, c = i & 15;
       const bool ok = r < qrows;
       const int qr = qr0 + (ok ? r : 0);
@@ -117,190 +131,215 @@ __global__ void __launch_bounds__(128) k_attn_bf16(const AttnParams a) {
       const bf16* src = Q + ((size_t)(ch.row0 + t) * a.Hq + u.kvh * G + g) * HD + c * 8;
       cp_async16(smem_u32(sQ) + swz(r, c), src, ok);
     }
-    if (tid < kAttnQRows) s_rowpos[tid] = (tid < qrows) ? ch.pos0 + (qr0 + tid) / G : -1;
-    for (int sb = 0; sb < NSUB; ++sb) {
-      for (int i = tid; i < SUB * 16; i += 128) {
-        const int r = i >> 4, c = i & 15;
-        const int kp = kp0 + sb * SUB + r;
-        const bf16* kr = key_row(a, Kp, Ki, ch, u.kvh, kp, max_kp);
-        const bf16* vr = key_row(a, Vp, Vi, ch, u.kvh, kp, max_kp);
-        cp_async16(smem_u32(sK + sb * TILE_BYTES) + swz(r, c), kr ? kr + c * 8 : Kp, kr != nullptr);
-        cp_async16(smem_u32(sV + sb * TILE_BYTES) + swz(r, c), vr ? vr + c * 8 : Vp, vr != nullptr);
-      }
-      cp_async_commit();
+    __syncthreads();  // page ids visible
+    // stage the chunk's keys and values
+    for (int i = tid; i < NSUB * SUB * 16; i += ATT_THREADS) {
+      const int r = i >> 4, c = i & 15;      // r: key within the chunk
+      const int kp = kp0 + r;
+      const bf16* kr = key_row(a, Kp, Ki, ch, u.kvh, kp, max_kp, kp0, s_page);
+      const bf16* vr = key_row(a, Vp, Vi, ch, u.kvh, kp, max_kp, kp0, s_page);
+      const int b = r / SUB, rr = r % SUB;
+      cp_async16(smem_u32(sK + b * TILE_BYTES) + swz(rr, c), kr ? kr + c * 8 : Kp, kr != nullptr);
+      cp_async16(smem_u32(sV + b * TILE_BYTES) + swz(rr, c), vr ? vr + c * 8 : Vp, vr != nullptr);
     }
-    cp_async_wait<NSUB - 1>();
+    cp_async_commit();
+    cp_async_wait<0>();
     __syncthreads();
 
     // Q fragments of this warp's 16 rows
     uint32_t qf[HD / 16][4];
 #pragma unroll
     for (int kk = 0; kk < HD / 16; ++kk) {
-      const int r = warp * 16 + (lane & 15), c = kk * 2 + (lane >> 4);
+      const int r = rg * 16 + (lane & 15), c = kk * 2 + (lane >> 4);
       ldsm_x4(smem_u32(sQ) + swz(r, c), qf[kk][0], qf[kk][1], qf[kk][2], qf[kk][3]);
     }
-    const int r_lo = warp * 16 + (lane >> 2), r_hi = r_lo + 8;
+    const int r_lo = rg * 16 + (lane >> 2), r_hi = r_lo + 8;
     const int pos_lo = s_rowpos[r_lo], pos_hi = s_rowpos[r_hi];
-    float m_lo = -INFINITY, m_hi = -INFINITY, l_lo = 0.f, l_hi = 0.f;
     float o[HD / 8][4];
 #pragma unroll
     for (int i = 0; i < HD / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
 
-#pragma unroll 1
-    for (int sb = 0; sb < NSUB; ++sb) {
-      if (sb == 1) {
-        cp_async_wait<0>();
-        __syncthreads();
-      }
-      const uint32_t kb = smem_u32(sK + sb * TILE_BYTES), vb = smem_u32(sV + sb * TILE_BYTES);
-      float s[SUB / 8][4];
+    const uint32_t kb = smem_u32(sK + sb * TILE_BYTES), vb = smem_u32(sV + sb * TILE_BYTES);
+    float s[SUB / 8][4];
 #pragma unroll
-      for (int nt = 0; nt < SUB / 8; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+    for (int nt = 0; nt < SUB / 8; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
 #pragma unroll
-      for (int kk = 0; kk < HD / 16; ++kk) {
+    for (int kk = 0; kk < HD / 16; ++kk) {
 #pragma unroll
-        for (int np = 0; np < SUB / 16; ++np) {
-          uint32_t b0, b1, b2, b3;
-          const int r = np * 16 + (lane & 7) + ((lane >> 4) << 3), c = kk * 2 + ((lane >> 3) & 1);
-          ldsm_x4(kb + swz(r, c), b0, b1, b2, b3);
-          mma16816(s[2 * np], qf[kk], b0, b1);
-          mma16816(s[2 * np + 1], qf[kk], b2, b3);
-        }
-      }
-      // mask (key position <= row position) and online softmax in the log2 domain
-      const int kbase = kp0 + sb * SUB + 2 * (lane & 3);
-      float mx_lo = m_lo, mx_hi = m_hi;
-#pragma unroll
-      for (int nt = 0; nt < SUB / 8; ++nt) {
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-          const int kp = kbase + nt * 8 + e;
-          s[nt][e] = (kp <= pos_lo) ? s[nt][e] * a.scale_log2 : -INFINITY;
-          s[nt][2 + e] = (kp <= pos_hi) ? s[nt][2 + e] * a.scale_log2 : -INFINITY;
-          mx_lo = fmaxf(mx_lo, s[nt][e]);
-          mx_hi = fmaxf(mx_hi, s[nt][2 + e]);
-        }
-      }
-#pragma unroll
-      for (int sh = 1; sh <= 2; sh <<= 1) {
-        mx_lo = fmaxf(mx_lo, __shfl_xor_sync(0xffffffffu, mx_lo, sh));
-        mx_hi = fmaxf(mx_hi, __shfl_xor_sync(0xffffffffu, mx_hi, sh));
-      }
-      const float al_lo = (mx_lo == -INFINITY) ? 1.f : exp2f(m_lo - mx_lo);
-      const float al_hi = (mx_hi == -INFINITY) ? 1.f : exp2f(m_hi - mx_hi);
-      const float b_lo = (mx_lo == -INFINITY) ? 0.f : mx_lo;
-      const float b_hi = (mx_hi == -INFINITY) ? 0.f : mx_hi;
-      m_lo = mx_lo;
-      m_hi = mx_hi;
-      float ps_lo = 0.f, ps_hi = 0.f;
-#pragma unroll
-      for (int nt = 0; nt < SUB / 8; ++nt) {
-        s[nt][0] = exp2f(s[nt][0] - b_lo);
-        s[nt][1] = exp2f(s[nt][1] - b_lo);
-        s[nt][2] = exp2f(s[nt][2] - b_hi);
-        s[nt][3] = exp2f(s[nt][3] - b_hi);
-        ps_lo += s[nt][0] + s[nt][1];
-        ps_hi += s[nt][2] + s[nt][3];
-      }
-      l_lo = l_lo * al_lo + ps_lo;
-      l_hi = l_hi * al_hi + ps_hi;
-#pragma unroll
-      for (int i = 0; i < HD / 8; ++i) {
-        o[i][0] *= al_lo;
-        o[i][1] *= al_lo;
-        o[i][2] *= al_hi;
-        o[i][3] *= al_hi;
-      }
-      // O += P V
-#pragma unroll
-      for (int kj = 0; kj < SUB / 16; ++kj) {
-        uint32_t pa[4];
-        pa[0] = pack_bf16(s[2 * kj][0], s[2 * kj][1]);
-        pa[1] = pack_bf16(s[2 * kj][2], s[2 * kj][3]);
-        pa[2] = pack_bf16(s[2 * kj + 1][0], s[2 * kj + 1][1]);
-        pa[3] = pack_bf16(s[2 * kj + 1][2], s[2 * kj + 1][3]);
-#pragma unroll
-        for (int dp = 0; dp < HD / 16; ++dp) {
-          uint32_t b0, b1, b2, b3;
-          const int r = kj * 16 + (lane & 7) + (((lane >> 3) & 1) << 3), c = dp * 2 + (lane >> 4);
-          ldsm_x4_t(vb + swz(r, c), b0, b1, b2, b3);
-          mma16816(o[2 * dp], pa, b0, b1);
-          mma16816(o[2 * dp + 1], pa, b2, b3);
-        }
+      for (int np = 0; np < SUB / 16; ++np) {
+        uint32_t b0, b1, b2, b3;
+        const int r = np * 16 + (lane & 7) + ((lane >> 4) << 3), c = kk * 2 + ((lane >> 3) & 1);
+        ldsm_x4(kb + swz(r, c), b0, b1, b2, b3);
+        mma16816(s[2 * np], qf[kk], b0, b1);
+        mma16816(s[2 * np + 1], qf[kk], b2, b3);
       }
     }
-    // row sums across the quad
+    // mask (key position <= row position); softmax statistics of this 64-key sub-block (log2 domain)
+    const int kbase = kp0 + sb * SUB + 2 * (lane & 3);
+    float m_lo = -INFINITY, m_hi = -INFINITY;
+#pragma unroll
+    for (int nt = 0; nt < SUB / 8; ++nt) {
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const int kp = kbase + nt * 8 + e;
+        s[nt][e] = (kp <= pos_lo) ? s[nt][e] * a.scale_log2 : -INFINITY;
+        s[nt][2 + e] = (kp <= pos_hi) ? s[nt][2 + e] * a.scale_log2 : -INFINITY;
+        m_lo = fmaxf(m_lo, s[nt][e]);
+        m_hi = fmaxf(m_hi, s[nt][2 + e]);
+      }
+    }
+#pragma unroll
+    for (int sh = 1; sh <= 2; sh <<= 1) {
+      m_lo = fmaxf(m_lo, __shfl_xor_sync(0xffffffffu, m_lo, sh));
+      m_hi = fmaxf(m_hi, __shfl_xor_sync(0xffffffffu, m_hi, sh));
+    }
+    const float b_lo = (m_lo == -INFINITY) ? 0.f : m_lo;
+    const float b_hi = (m_hi == -INFINITY) ? 0.f : m_hi;
+    float l_lo = 0.f, l_hi = 0.f;
+#pragma unroll
+    for (int nt = 0; nt < SUB / 8; ++nt) {
+      s[nt][0] = exp2f(s[nt][0] - b_lo);
+      s[nt][1] = exp2f(s[nt][1] - b_lo);
+      s[nt][2] = exp2f(s[nt][2] - b_hi);
+      s[nt][3] = exp2f(s[nt][3] - b_hi);
+      l_lo += s[nt][0] + s[nt][1];
+      l_hi += s[nt][2] + s[nt][3];
+    }
+    // O = P V
+#pragma unroll
+    for (int kj = 0; kj < SUB / 16; ++kj) {
+      uint32_t pa[4];
+      pa[0] = pack_bf16(s[2 * kj][0], s[2 * kj][1]);
+      pa[1] = pack_bf16(s[2 * kj][2], s[2 * kj][3]);
+      pa[2] = pack_bf16(s[2 * kj + 1][0], s[2 * kj + 1][1]);
+      pa[3] = pack_bf16(s[2 * kj + 1][2], s[2 * kj + 1][3]);
+#pragma unroll
+      for (int dp = 0; dp < HD / 16; ++dp) {
+        uint32_t b0, b1, b2, b3;
+        const int r = kj * 16 + (lane & 7) + (((lane >> 3) & 1) << 3), c = dp * 2 + (lane >> 4);
+        ldsm_x4_t(vb + swz(r, c), b0, b1, b2, b3);
+        mma16816(o[2 * dp], pa, b0, b1);
+        mma16816(o[2 * dp + 1], pa, b2, b3);
+      }
+    }
 #pragma unroll
     for (int sh = 1; sh <= 2; sh <<= 1) {
       l_lo += __shfl_xor_sync(0xffffffffu, l_lo, sh);
       l_hi += __shfl_xor_sync(0xffffffffu, l_hi, sh);
     }
     const int d0 = 2 * (lane & 3);
-    if (u.n_chunks == 1) {
-      const float il_lo = l_lo > 0.f ? 1.f / l_lo : 0.f, il_hi = l_hi > 0.f ? 1.f / l_hi : 0.f;
-#pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        const int r = half ? r_hi : r_lo;
-        if (r >= qrows) continue;
-        const float il = half ? il_hi : il_lo;
-        const int qr = qr0 + r, t = qr / G, g = qr % G;
-        bf16* dst = Out + ((size_t)(ch.row0 + t) * a.Hq + u.kvh * G + g) * HD;
-#pragma unroll
-        for (int i = 0; i < HD / 8; ++i) {
-          const float x0 = o[i][2 * half] * il, x1 = o[i][2 * half + 1] * il;
-          *reinterpret_cast<uint32_t*>(dst + i * 8 + d0) = pack_bf16(x0, x1);
-        }
-      }
-    } else {
-      const int slot = u.slot0 + chunk;
-      float* wo = a.ws_o + (size_t)slot * kAttnQRows * HD;
-      float* wml = a.ws_ml + (size_t)slot * kAttnQRows * 2;
+    __syncthreads();  // every warp is done with K/V: sub-block 1 partials may overwrite them
+    if (sb == 1) {
 #pragma unroll
       for (int i = 0; i < HD / 8; ++i) {
-        *reinterpret_cast<float2*>(wo + r_lo * HD + i * 8 + d0) = make_float2(o[i][0], o[i][1]);
-        *reinterpret_cast<float2*>(wo + r_hi * HD + i * 8 + d0) = make_float2(o[i][2], o[i][3]);
+        *reinterpret_cast<float2*>(sO1 + r_lo * HD + i * 8 + d0) = make_float2(o[i][0], o[i][1]);
+        *reinterpret_cast<float2*>(sO1 + r_hi * HD + i * 8 + d0) = make_float2(o[i][2], o[i][3]);
       }
       if ((lane & 3) == 0) {
-        wml[r_lo * 2] = m_lo;
-        wml[r_lo * 2 + 1] = l_lo;
-        wml[r_hi * 2] = m_hi;
-        wml[r_hi * 2 + 1] = l_hi;
+        s_m1[r_lo] = m_lo;
+        s_l1[r_lo] = l_lo;
+        s_m1[r_hi] = m_hi;
+        s_l1[r_hi] = l_hi;
       }
-      __threadfence();
-      __syncthreads();
-      if (tid == 0) s_last = (atomicAdd(a.unit_counter + it.x, 1) == u.n_chunks - 1);
-      __syncthreads();
-      if (s_last) {
-        __threadfence();
-        // merge the unit's chunks in chunk order: out = sum_c 2^(m_c - M) O_c / sum_c 2^(m_c - M) l_c
-        for (int i = tid; i < qrows * (HD / 4); i += 128) {
-          const int r = i / (HD / 4), d = (i % (HD / 4)) * 4;
-          float M = -INFINITY;
-          for (int c = 0; c < u.n_chunks; ++c) M = fmaxf(M, __ldcg(a.ws_ml + ((size_t)(u.slot0 + c) * kAttnQRows + r) * 2));
-          float L = 0.f, acc0 = 0.f, acc1 = 0.f, acc2 = 0.f, acc3 = 0.f;
-          for (int c = 0; c < u.n_chunks; ++c) {
-            const size_t sl = (size_t)(u.slot0 + c);
-            const float mc = __ldcg(a.ws_ml + (sl * kAttnQRows + r) * 2);
-            const float w = (mc == -INFINITY) ? 0.f : exp2f(mc - M);
-            L += w * __ldcg(a.ws_ml + (sl * kAttnQRows + r) * 2 + 1);
-            const float4 oc = __ldcg(reinterpret_cast<const float4*>(a.ws_o + (sl * kAttnQRows + r) * HD + d));
-            acc0 += w * oc.x;
-            acc1 += w * oc.y;
-            acc2 += w * oc.z;
-            acc3 += w * oc.w;
-          }
-          const float il = L > 0.f ? 1.f / L : 0.f;
+    }
+    __syncthreads();
+    if (sb == 0) {
+      // merge: m = max(m0, m1), O = 2^(m0-m) O0 + 2^(m1-m) O1, l likewise
+      const float m1_lo = s_m1[r_lo], m1_hi = s_m1[r_hi];
+      const float mm_lo = fmaxf(m_lo, m1_lo), mm_hi = fmaxf(m_hi, m1_hi);
+      const float a0_lo = (m_lo == -INFINITY) ? 0.f : exp2f(m_lo - mm_lo);
+      const float a1_lo = (m1_lo == -INFINITY) ? 0.f : exp2f(m1_lo - mm_lo);
+      const float a0_hi = (m_hi == -INFINITY) ? 0.f : exp2f(m_hi - mm_hi);
+      const float a1_hi = (m1_hi == -INFINITY) ? 0.f : exp2f(m1_hi - mm_hi);
+      l_lo = a0_lo * l_lo + a1_lo * s_l1[r_lo];
+      l_hi = a0_hi * l_hi + a1_hi * s_l1[r_hi];
+#pragma unroll
+      for (int i = 0; i < HD / 8; ++i) {
+        const float2 p_lo = *reinterpret_cast<const float2*>(sO1 + r_lo * HD + i * 8 + d0);
+        const float2 p_hi = *reinterpret_cast<const float2*>(sO1 + r_hi * HD + i * 8 + d0);
+        o[i][0] = a0_lo * o[i][0] + a1_lo * p_lo.x;
+        o[i][1] = a0_lo * o[i][1] + a1_lo * p_lo.y;
+        o[i][2] = a0_hi * o[i][2] + a1_hi * p_hi.x;
+        o[i][3] = a0_hi * o[i][3] + a1_hi * p_hi.y;
+      }
+      m_lo = mm_lo;
+      m_hi = mm_hi;
+      if (u.n_chunks == 1) {
+        const float il_lo = l_lo > 0.f ? 1.f / l_lo : 0.f, il_hi = l_hi > 0.f ? 1.f / l_hi : 0.f;
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+          const int r = half ? r_hi : r_lo;
+          if (r >= qrows) continue;
+          const float il = half ? il_hi : il_lo;
           const int qr = qr0 + r, t = qr / G, g = qr % G;
-          bf16* dst = Out + ((size_t)(ch.row0 + t) * a.Hq + u.kvh * G + g) * HD + d;
-          *reinterpret_cast<uint32_t*>(dst) = pack_bf16(acc0 * il, acc1 * il);
-          *reinterpret_cast<uint32_t*>(dst + 2) = pack_bf16(acc2 * il, acc3 * il);
+          bf16* dst = Out + ((size_t)(ch.row0 + t) * a.Hq + u.kvh * G + g) * HD;
+#pragma unroll
+          for (int i = 0; i < HD / 8; ++i) {
+            const float x0 = o[i][2 * half] * il, x1 = o[i][2 * half + 1] * il;
+            *reinterpret_cast<uint32_t*>(dst + i * 8 + d0) = pack_bf16(x0, x1);
+          }
         }
-        if (tid == 0) a.unit_counter[it.x] = 0;
+      } else {
+        const int slot = u.slot0 + chunk;
+        float* wo = a.ws_o + (size_t)slot * kAttnQRows * HD;
+        float* wml = a.ws_ml + (size_t)slot * kAttnQRows * 2;
+#pragma unroll
+        for (int i = 0; i < HD / 8; ++i) {
+          *reinterpret_cast<float2*>(wo + r_lo * HD + i * 8 + d0) = make_float2(o[i][0], o[i][1]);
+          *reinterpret_cast<float2*>(wo + r_hi * HD + i * 8 + d0) = make_float2(o[i][2], o[i][3]);
+        }
+        if ((lane & 3) == 0) {
+          wml[r_lo * 2] = m_lo;
+          wml[r_lo * 2 + 1] = l_lo;
+          wml[r_hi * 2] = m_hi;
+          wml[r_hi * 2 + 1] = l_hi;
+        }
       }
     }
     __syncthreads();
   }
+}
+
+// Merge of the split-KV partials of multi-chunk units, in chunk order:
+//   out = sum_c 2^(m_c - M) O_c / sum_c 2^(m_c - M) l_c,  M = max_c m_c.
+// CTA (x, u) handles rows 8x .. 8x+7 of unit u; thread = (row, 4 of the 128 dims).
+__global__ void __launch_bounds__(256) k_attn_combine(const AttnParams a) {
   pdl_launch_dependents();
+  pdl_wait();
+  const int u_idx = blockIdx.y;
+  if (u_idx >= a.plan->n_units) return;
+  const AttnUnit u = a.units[u_idx];
+  if (u.n_chunks == 1) return;
+  const Chain ch = a.chains[u.chain];
+  const int G = a.Hq / a.Hkv;
+  const int qr0 = u.qt * kAttnQRows;
+  int qrows = ch.nrows * G - qr0;
+  if (qrows > kAttnQRows) qrows = kAttnQRows;
+  const int r = blockIdx.x * 8 + (threadIdx.x >> 5);
+  if (r >= qrows) return;
+  const int d = (threadIdx.x & 31) * 4;
+  const float2* ml = reinterpret_cast<const float2*>(a.ws_ml);
+  float M = -INFINITY;
+#pragma unroll 4
+  for (int c = 0; c < u.n_chunks; ++c) M = fmaxf(M, __ldcg(ml + (size_t)(u.slot0 + c) * kAttnQRows + r).x);
+  float L = 0.f, acc0 = 0.f, acc1 = 0.f, acc2 = 0.f, acc3 = 0.f;
+#pragma unroll 4
+  for (int c = 0; c < u.n_chunks; ++c) {
+    const size_t sl = (size_t)(u.slot0 + c);
+    const float2 p = __ldcg(ml + sl * kAttnQRows + r);
+    const float4 oc = __ldcg(reinterpret_cast<const float4*>(a.ws_o + (sl * kAttnQRows + r) * HD + d));
+    const float w = (p.x == -INFINITY) ? 0.f : exp2f(p.x - M);
+    L += w * p.y;
+    acc0 += w * oc.x;
+    acc1 += w * oc.y;
+    acc2 += w * oc.z;
+    acc3 += w * oc.w;
+  }
+  const float il = L > 0.f ? 1.f / L : 0.f;
+  const int qr = qr0 + r, t = qr / G, g = qr % G;
+  bf16* dst = reinterpret_cast<bf16*>(a.out) + ((size_t)(ch.row0 + t) * a.Hq + u.kvh * G + g) * HD + d;
+  *reinterpret_cast<uint32_t*>(dst) = pack_bf16(acc0 * il, acc1 * il);
+  *reinterpret_cast<uint32_t*>(dst + 2) = pack_bf16(acc2 * il, acc3 * il);
 }
 
 // fp32 path: one warp per (row, query head); keys in absolute order, 32 at a time.
@@ -382,6 +421,7 @@ __global__ void __launch_bounds__(128) k_attn_f32(const AttnParams a, int n_rows
 // Work decomposition of the bf16 attention for the current chains (one CTA, once per forward).
 __global__ void k_attn_plan(const Chain* chains, const int* n_chains_dev, int Hq, int Hkv, AttnPlan* plan,
                             AttnUnit* units, int2* items, int max_units, int max_items, int max_slots, int* err) {
+  pdl_launch_dependents();
   pdl_wait();
   if (threadIdx.x != 0) return;
   const int G = Hq / Hkv;
@@ -442,7 +482,7 @@ cudaError_t launch_attn_bf16(const AttnParams& a, int grid, cudaStream_t st) {
   const size_t smem = attn_bf16_smem_bytes();
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
-  cfg.blockDim = dim3(128);
+  cfg.blockDim = dim3(ATT_THREADS);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = st;
   cudaLaunchAttribute at[1];
@@ -451,6 +491,19 @@ cudaError_t launch_attn_bf16(const AttnParams& a, int grid, cudaStream_t st) {
   cfg.attrs = at;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, k_attn_bf16, a);
+}
+
+cudaError_t launch_attn_combine(const AttnParams& a, int max_units, cudaStream_t st) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(kAttnQRows / 8, max_units);
+  cfg.blockDim = dim3(256);
+  cfg.stream = st;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, k_attn_combine, a);
 }
 
 cudaError_t launch_attn_f32(const AttnParams& a, int n_rows, cudaStream_t st) {

@@ -66,6 +66,7 @@ __global__ void k_rope_table(float2* tab, int n_pos, int half, double theta) {
 template <typename T>
 __global__ void k_embed(const T* __restrict__ E, const int* __restrict__ tok, float* __restrict__ x, int d, int V,
                         int* err) {
+  pdl_launch_dependents();
   pdl_wait();
   const int r = blockIdx.x;
   int t = tok[r];
@@ -76,29 +77,60 @@ __global__ void k_embed(const T* __restrict__ E, const int* __restrict__ tok, fl
   const T* src = E + (size_t)t * d;
   float* dst = x + (size_t)r * d;
   for (int i = threadIdx.x; i < d; i += blockDim.x) dst[i] = act_to_f32(src[i]);
-  pdl_launch_dependents();
 }
 
 // y[r, :] = x[r, :] / sqrt(mean(x[r, :]^2) + eps) * gain, rounded to the activation type.
+// One CTA per row; the row stays in registers (float4, up to 8 per thread: d <= 8192), so x is
+// read once. The reduction order is fixed by d alone.
+constexpr int NORM_THREADS = 256;
+constexpr int NORM_VEC = 8;
+
+__device__ __forceinline__ void store4(float* y, float4 v) { *reinterpret_cast<float4*>(y) = v; }
+__device__ __forceinline__ void store4(bf16* y, float4 v) {
+  const uint32_t lo = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.x)) |
+                      ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.y)) << 16);
+  const uint32_t hi = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.z)) |
+                      ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.w)) << 16);
+  *reinterpret_cast<uint2*>(y) = make_uint2(lo, hi);
+}
+
 template <typename T>
-__global__ void __launch_bounds__(256) k_rmsnorm(const float* __restrict__ x, const float* __restrict__ gain,
-                                                 T* __restrict__ y, int d, float eps) {
-  __shared__ float red[8];
+__global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(const float* __restrict__ x, const float* __restrict__ gain,
+                                                          T* __restrict__ y, int d, float eps) {
+  __shared__ float red[NORM_THREADS / 32];
+  pdl_launch_dependents();  // the next projection may launch now and prefetch its weights
   pdl_wait();
   const int r = blockIdx.x;
-  const float* xr = x + (size_t)r * d;
+  const int nv = d >> 2;
+  const float4* xr = reinterpret_cast<const float4*>(x + (size_t)r * d);
+  float4 v[NORM_VEC];
   float ss = 0.f;
-  for (int i = threadIdx.x; i < d; i += 256) ss = fmaf(xr[i], xr[i], ss);
+#pragma unroll
+  for (int j = 0; j < NORM_VEC; ++j) {
+    const int i = threadIdx.x + j * NORM_THREADS;
+    v[j] = (i < nv) ? xr[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+    ss = fmaf(v[j].x, v[j].x, ss);
+    ss = fmaf(v[j].y, v[j].y, ss);
+    ss = fmaf(v[j].z, v[j].z, ss);
+    ss = fmaf(v[j].w, v[j].w, ss);
+  }
   ss = warp_sum(ss);
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
   __syncthreads();
   float tot = 0.f;
 #pragma unroll
-  for (int w = 0; w < 8; ++w) tot += red[w];
+  for (int w = 0; w < NORM_THREADS / 32; ++w) tot += red[w];
   const float rs = 1.0f / sqrtf(tot / (float)d + eps);
+  const float4* g4 = reinterpret_cast<const float4*>(gain);
   T* yr = y + (size_t)r * d;
-  for (int i = threadIdx.x; i < d; i += 256) yr[i] = to_act<T>(xr[i] * rs * gain[i]);
-  pdl_launch_dependents();
+#pragma unroll
+  for (int j = 0; j < NORM_VEC; ++j) {
+    const int i = threadIdx.x + j * NORM_THREADS;
+    if (i < nv) {
+      const float4 g = g4[i];
+      store4(yr + 4 * i, make_float4(v[j].x * rs * g.x, v[j].y * rs * g.y, v[j].z * rs * g.z, v[j].w * rs * g.w));
+    }
+  }
 }
 
 template <typename K, typename... Args>
@@ -158,8 +190,8 @@ cudaError_t launch_embed(const void* E, bool is_bf16, const int* tok, float* x, 
 cudaError_t launch_rmsnorm(const float* x, const float* gain, void* y, bool is_bf16, int rows, int d, float eps,
                            cudaStream_t st) {
   if (is_bf16)
-    return launch_pdl(k_rmsnorm<bf16>, dim3(rows), dim3(256), st, x, gain, reinterpret_cast<bf16*>(y), d, eps);
-  return launch_pdl(k_rmsnorm<float>, dim3(rows), dim3(256), st, x, gain, reinterpret_cast<float*>(y), d, eps);
+    return launch_pdl(k_rmsnorm<bf16>, dim3(rows), dim3(NORM_THREADS), st, x, gain, reinterpret_cast<bf16*>(y), d, eps);
+  return launch_pdl(k_rmsnorm<float>, dim3(rows), dim3(NORM_THREADS), st, x, gain, reinterpret_cast<float*>(y), d, eps);
 }
 
 }  // namespace jf

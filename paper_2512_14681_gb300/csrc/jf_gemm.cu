@@ -36,29 +36,28 @@ JF_DEV uint8_t* align1024(uint8_t* p) {
 // Epilogue on one 16-column chunk: thread `row` (0..127) holds v[j] = Y[m0 + c0 + j, n0 + row].
 // xs: shared staging [16][128] fp32 (exchange between the two halves of a tile).
 // ---------------------------------------------------------------------------------------------
-template <typename T>
+template <typename T, int EPI>
 JF_DEV void epilogue_chunk(const GemmEpi& e, const float (&v)[16], int row, int n0, int m0, int c0, float* xs,
                            int n_tile, int n_tiles) {
   const int n = n0 + row;
-  const int kind = e.kind;
-  if (kind == EPI_STORE || kind == EPI_RESID) {
+  constexpr int kind = EPI;
+  if constexpr (kind == EPI_STORE || kind == EPI_RESID) {
     if (n < e.N) {
 #pragma unroll
       for (int j = 0; j < 16; ++j) {
         const int m = m0 + c0 + j;
         if (m < e.M) {
-          if (kind == EPI_STORE) e.y[(size_t)m * e.ldy + n] = v[j];
+          if constexpr (kind == EPI_STORE) e.y[(size_t)m * e.ldy + n] = v[j];
           else e.x[(size_t)m * e.ldx + n] += v[j];
         }
       }
     }
     return;
-  }
-  if (kind == EPI_QKV || kind == EPI_SWIGLU) {
+  } else if constexpr (kind == EPI_QKV || kind == EPI_SWIGLU) {
 #pragma unroll
     for (int j = 0; j < 16; ++j) xs[j * 128 + row] = v[j];
     __syncthreads();
-    if (kind == EPI_QKV) {
+    if constexpr (kind == EPI_QKV) {
       const int hd = e.head_dim, half = hd >> 1;
       const int i = n % hd;
       const bool is_q = n < e.n_q;
@@ -98,9 +97,8 @@ JF_DEV void epilogue_chunk(const GemmEpi& e, const float (&v)[16], int row, int 
     }
     __syncthreads();
     return;
-  }
-  // EPI_ARGMAX: best (value, index) and runner-up value over this tile's 128 vocabulary rows
-  {
+  } else {
+    // EPI_ARGMAX: best (value, index) and runner-up value over this tile's 128 vocabulary rows
     float* red = xs;  // [4 warps][16 cols][3]
     const int warp = row >> 5, lane = row & 31;
 #pragma unroll
@@ -176,7 +174,7 @@ JF_DEV void argmax_finish(const GemmEpi& e, int m0, int BN, int n_tiles, int tid
 
 // Shared tail of both mainloops: ticketing for split-K and argmax, then the epilogue.
 // get(c0, v) fills this thread's 16 accumulator values of columns c0..c0+15.
-template <typename T, int BN, typename Get>
+template <typename T, int BN, int EPI, typename Get>
 JF_DEV void finish_tile(const GemmParams& p, Get get, float* xs, int* sflag) {
   const int tid = threadIdx.x;
   const int n_tile = blockIdx.x, split = blockIdx.y, m_tile = blockIdx.z;
@@ -189,7 +187,7 @@ JF_DEV void finish_tile(const GemmParams& p, Get get, float* xs, int* sflag) {
     for (int c = 0; c < nchunks; ++c) {
       float v[16];
       get(c * 16, v);
-      epilogue_chunk<T>(p.epi, v, tid, n0, m0, c * 16, xs, n_tile, p.n_tiles);
+      epilogue_chunk<T, EPI>(p.epi, v, tid, n0, m0, c * 16, xs, n_tile, p.n_tiles);
     }
   } else {
     float* mine = p.ws + ((size_t)tile_lin * p.k_splits + split) * (size_t)BN * kTileN;
@@ -218,11 +216,11 @@ JF_DEV void finish_tile(const GemmParams& p, Get get, float* xs, int* sflag) {
 #pragma unroll
         for (int j = 0; j < 16; ++j) v[j] += __ldcg(src + (c * 16 + j) * kTileN + tid);
       }
-      epilogue_chunk<T>(p.epi, v, tid, n0, m0, c * 16, xs, n_tile, p.n_tiles);
+      epilogue_chunk<T, EPI>(p.epi, v, tid, n0, m0, c * 16, xs, n_tile, p.n_tiles);
     }
     if (tid == 0) p.tile_counter[tile_lin] = 0;
   }
-  if (p.epi.kind == EPI_ARGMAX) {
+  if constexpr (EPI == EPI_ARGMAX) {
     __threadfence();
     __syncthreads();
     if (tid == 0) {
@@ -242,7 +240,7 @@ JF_DEV void finish_tile(const GemmParams& p, Get get, float* xs, int* sflag) {
 // bf16 tcgen05 kernel. 128 threads: thread 0 = TMA producer, thread 32 = MMA issuer, then all
 // four warps drain the accumulator (warp w reads TMEM lanes 32w .. 32w+31).
 // ---------------------------------------------------------------------------------------------
-template <int BN>
+template <int BN, int EPI>
 __global__ void __launch_bounds__(128, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const GemmParams p) {
   using Cfg = TcCfg<BN>;
@@ -264,11 +262,11 @@ __global__ void __launch_bounds__(128, 1)
   const int nkb = kb_end - kb_begin;
   const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + S), accum = smem_u32(bars + 2 * S);
 
-  if (warp == 0) {
-    tmem_alloc(smem_u32(tmem_slot), Cfg::TMEM_COLS);
-    tmem_relinquish();
-  }
-  if (tid == 32) {
+  // thread 0 initialises the barriers and requests the first weight stages right away: weights do
+  // not depend on earlier kernels, so they stream in while TMEM is allocated and while the previous
+  // kernel of the chain finishes.
+  const int pre = nkb < S ? nkb : S;
+  if (tid == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(full0 + 8 * s, 1);
       mbar_init(empty0 + 8 * s, 1);
@@ -276,10 +274,18 @@ __global__ void __launch_bounds__(128, 1)
     mbar_init(accum, 1);
     *sok = 1;
     fence_mbar_init();
-  }
-  if (tid == 64) {
     tma_prefetch_desc(&tmA);
     tma_prefetch_desc(&tmB);
+    const uint64_t polA = l2_policy_evict_first();
+    for (int i = 0; i < pre; ++i) {
+      mbar_arrive_expect_tx(full0 + 8 * i, Cfg::STAGE_BYTES);
+      tma_load_2d(smem_u32(sA + i * A_STAGE_BYTES), &tmA, full0 + 8 * i, (kb_begin + i) * kTileK, n0, polA);
+    }
+  }
+  __syncwarp();
+  if (warp == 0) {
+    tmem_alloc(smem_u32(tmem_slot), Cfg::TMEM_COLS);
+    tmem_relinquish();
   }
   tc_fence_before();
   __syncthreads();
@@ -287,14 +293,8 @@ __global__ void __launch_bounds__(128, 1)
   const uint32_t tmem = *tmem_slot;
 
   if (tid == 0) {
-    // producer: weights do not depend on earlier kernels, so the first stages are requested
-    // before waiting for the previous kernel of the chain.
+    // producer: activations after the previous kernel has completed, then the steady state
     const uint64_t polA = l2_policy_evict_first(), polB = l2_policy_evict_last();
-    const int pre = nkb < S ? nkb : S;
-    for (int i = 0; i < pre; ++i) {
-      mbar_arrive_expect_tx(full0 + 8 * i, Cfg::STAGE_BYTES);
-      tma_load_2d(smem_u32(sA + i * A_STAGE_BYTES), &tmA, full0 + 8 * i, (kb_begin + i) * kTileK, n0, polA);
-    }
     pdl_wait();
     for (int i = 0; i < pre; ++i)
       tma_load_2d(smem_u32(sB + i * Cfg::B_STAGE_BYTES), &tmB, full0 + 8 * i, (kb_begin + i) * kTileK, m0, polB);
@@ -341,7 +341,7 @@ __global__ void __launch_bounds__(128, 1)
     float* xs = reinterpret_cast<float*>(sA);
     const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
     auto get = [&](int c0, float (&v)[16]) { tmem_ld16(tmem + lane_base + (uint32_t)c0, v); };
-    finish_tile<bf16, BN>(p, get, xs, sflag);
+    finish_tile<bf16, BN, EPI>(p, get, xs, sflag);
   }
   tc_fence_before();
   __syncthreads();
@@ -355,6 +355,7 @@ __global__ void __launch_bounds__(128, 1)
 constexpr int F32_BN = 32;
 constexpr int F32_BK = 32;
 
+template <int EPI>
 __global__ void __launch_bounds__(128) k_gemm_f32(const float* __restrict__ W, const float* __restrict__ X,
                                                   const GemmParams p) {
   __shared__ float xt[F32_BN][F32_BK + 1];
@@ -396,11 +397,11 @@ __global__ void __launch_bounds__(128) k_gemm_f32(const float* __restrict__ W, c
         for (int j = 0; j < 16; ++j) v[j] = acc[cc + j];
       }
   };
-  finish_tile<float, F32_BN>(p, get, xs, &sflag);
+  finish_tile<float, F32_BN, EPI>(p, get, xs, &sflag);
 }
 
-template <int BN>
-cudaError_t launch_tc(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmParams& p, cudaStream_t st) {
+template <int BN, int EPI>
+cudaError_t launch_tc_epi(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmParams& p, cudaStream_t st) {
   using Cfg = TcCfg<BN>;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.n_tiles, p.k_splits, p.m_tiles);
@@ -412,12 +413,30 @@ cudaError_t launch_tc(const CUtensorMap& tmA, const CUtensorMap& tmB, const Gemm
   at[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = at;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, k_gemm_tc<BN>, tmA, tmB, p);
+  return cudaLaunchKernelEx(&cfg, k_gemm_tc<BN, EPI>, tmA, tmB, p);
+}
+
+template <int BN>
+cudaError_t launch_tc(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmParams& p, cudaStream_t st) {
+  switch (p.epi.kind) {
+    case EPI_STORE: return launch_tc_epi<BN, EPI_STORE>(tmA, tmB, p, st);
+    case EPI_RESID: return launch_tc_epi<BN, EPI_RESID>(tmA, tmB, p, st);
+    case EPI_QKV: return launch_tc_epi<BN, EPI_QKV>(tmA, tmB, p, st);
+    case EPI_SWIGLU: return launch_tc_epi<BN, EPI_SWIGLU>(tmA, tmB, p, st);
+    case EPI_ARGMAX: return launch_tc_epi<BN, EPI_ARGMAX>(tmA, tmB, p, st);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 template <int BN>
 cudaError_t prep_tc() {
-  return cudaFuncSetAttribute(k_gemm_tc<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<BN>::SMEM);
+  cudaError_t e;
+  const int sm = TcCfg<BN>::SMEM;
+  if ((e = cudaFuncSetAttribute(k_gemm_tc<BN, EPI_STORE>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm))) return e;
+  if ((e = cudaFuncSetAttribute(k_gemm_tc<BN, EPI_RESID>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm))) return e;
+  if ((e = cudaFuncSetAttribute(k_gemm_tc<BN, EPI_QKV>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm))) return e;
+  if ((e = cudaFuncSetAttribute(k_gemm_tc<BN, EPI_SWIGLU>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm))) return e;
+  return cudaFuncSetAttribute(k_gemm_tc<BN, EPI_ARGMAX>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
 }
 
 }  // namespace
@@ -477,7 +496,14 @@ cudaError_t launch_gemm_f32(const float* W, const float* X, const GemmParams& p,
   at[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = at;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, k_gemm_f32, W, X, p);
+  switch (p.epi.kind) {
+    case EPI_STORE: return cudaLaunchKernelEx(&cfg, k_gemm_f32<EPI_STORE>, W, X, p);
+    case EPI_RESID: return cudaLaunchKernelEx(&cfg, k_gemm_f32<EPI_RESID>, W, X, p);
+    case EPI_QKV: return cudaLaunchKernelEx(&cfg, k_gemm_f32<EPI_QKV>, W, X, p);
+    case EPI_SWIGLU: return cudaLaunchKernelEx(&cfg, k_gemm_f32<EPI_SWIGLU>, W, X, p);
+    case EPI_ARGMAX: return cudaLaunchKernelEx(&cfg, k_gemm_f32<EPI_ARGMAX>, W, X, p);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 }  // namespace jf

@@ -29,6 +29,7 @@ cudaError_t launch_attn_plan(const Chain* chains, const int* n_chains_dev, int H
                              cudaStream_t st);
 cudaError_t launch_attn_bf16(const AttnParams& a, int grid, cudaStream_t st);
 cudaError_t launch_attn_f32(const AttnParams& a, int n_rows, cudaStream_t st);
+cudaError_t launch_attn_combine(const AttnParams& a, int max_units, cudaStream_t st);
 size_t attn_bf16_smem_bytes();
 cudaError_t gemm_prepare();
 cudaError_t attn_prepare();
@@ -39,6 +40,11 @@ using namespace jf;
 namespace {
 
 constexpr int kTargetCTAs = 152;   // split-K target: about one CTA per SM of a GB300
+// kernel classes of jf_kernel_time (include/jf.h)
+enum ProfClass : int {
+  PC_GATEUP = 0, PC_ATTN = 1, PC_GEMMS = 2, PC_QKV = 3, PC_OPROJ = 4, PC_DOWN = 5, PC_LMHEAD = 6, PC_COMBINE = 7,
+  PC_NORM = 8, PC_OTHER = 9, kProfClasses = 10
+};
 constexpr int kMaxStateInts = 32768;
 constexpr int kRandomTidMax = 8 + 16 * 4096;
 
@@ -130,6 +136,7 @@ jf_status make_dims(const jf_model_config* m, const jf_runtime_config* rt, Dims*
     return JF_EUNSUPPORTED;
   }
   if (m->d_model % 64 || m->d_ff % 64) { *why = "d_model and d_ff must be multiples of 64"; return JF_EUNSUPPORTED; }
+  if (m->d_model > 8192) { *why = "d_model above 8192 is not supported by the norm kernel"; return JF_EUNSUPPORTED; }
   if (rt->max_seqs < 1 || rt->max_seqs > kMaxSeqs || rt->max_ctx < 16 || rt->max_rows < 1 || rt->max_rows > 4096 ||
       rt->logits_rows < 0 || rt->logits_rows > rt->max_rows) {
     *why = "runtime capacity out of range (max_seqs 1..64, max_ctx >= 16, max_rows 1..4096, logits_rows <= max_rows)";
@@ -264,6 +271,7 @@ struct jf_ctx {
   cudaStream_t st = nullptr;
   bool own_stream = false;
   int device = 0;
+  int num_sms = 152;
   std::string last_error;
   bool weights_ready = false;
   // device pointers
@@ -310,8 +318,8 @@ struct jf_ctx {
   bool have_graph_cfg = false;
   // profiling
   bool profiling = false;
-  double prof_ms[3] = {0, 0, 0};
-  long long prof_n[3] = {0, 0, 0};
+  double prof_ms[kProfClasses] = {};
+  long long prof_n[kProfClasses] = {};
   std::vector<cudaEvent_t>* capture_events = nullptr;
   std::vector<int>* capture_classes = nullptr;
   long long launches = 0;  // libjf kernels launched (graph replays count their kernel nodes)
@@ -409,7 +417,9 @@ jf_status set_seq_len(jf_ctx* c, int seq, int len) {
 // ------------------------------------------------------------------------------------------
 // Forward pass launch sequence (one pass over M in-flight rows; Eq. 3).
 // ------------------------------------------------------------------------------------------
-enum LmMode { LM_ARGMAX = 0, LM_LOGITS = 1 };
+// LM head of a forward: greedy argmax of every row, logits of every row, argmax of the last row
+// only (prefill: only the token after the prompt is needed), or none (non-final prefill chunks).
+enum LmMode { LM_ARGMAX = 0, LM_LOGITS = 1, LM_LAST = 2, LM_NONE = 3 };
 
 void prof_begin(jf_ctx* c, int cls) {
   if (!c->capture_events) return;
@@ -441,7 +451,7 @@ cudaError_t gemm(jf_ctx* c, const CUtensorMap& tmA, const void* W, const void* X
   p.epi = epi;
   p.epi.M = M;
   p.epi.N = N;
-  const bool pr = c->capture_events && (cls == 0 || cls == 2);
+  const bool pr = c->capture_events && cls >= 0;
   if (pr) prof_begin(c, cls);
   cudaError_t e;
   if (D.bf16) {
@@ -464,10 +474,15 @@ cudaError_t enqueue_forward(jf_ctx* c, int M, LmMode lm) {
   const Dims& D = c->D;
   const float eps = (float)c->mc.rms_eps;
   cudaError_t e;
-  if ((e = launch_embed(c->w_embed, D.bf16, c->tok, c->x, M, D.d, D.V, c->err, c->st)) != cudaSuccess) return e;
+  prof_begin(c, PC_OTHER);
+  e = launch_embed(c->w_embed, D.bf16, c->tok, c->x, M, D.d, D.V, c->err, c->st);
+  prof_end(c);
+  if (e != cudaSuccess) return e;
   if (D.bf16) {
+    prof_begin(c, PC_OTHER);
     e = launch_attn_plan(c->chains, c->n_chains, D.Hq, D.Hkv, c->plan, c->units, c->items, D.max_units, D.max_items,
                          D.max_slots, c->err, c->st);
+    prof_end(c);
     if (e != cudaSuccess) return e;
   }
   const size_t inf_layer = (size_t)D.R * D.nkv * D.es;
@@ -476,13 +491,16 @@ cudaError_t enqueue_forward(jf_ctx* c, int M, LmMode lm) {
     LayerW& w = c->layers[l];
     char* kinf = reinterpret_cast<char*>(c->k_inf) + l * inf_layer;
     char* vinf = reinterpret_cast<char*>(c->v_inf) + l * inf_layer;
-    if ((e = launch_rmsnorm(c->x, w.g_attn, c->h, D.bf16, M, D.d, eps, c->st)) != cudaSuccess) return e;
+    prof_begin(c, PC_NORM);
+    e = launch_rmsnorm(c->x, w.g_attn, c->h, D.bf16, M, D.d, eps, c->st);
+    prof_end(c);
+    if (e != cudaSuccess) return e;
     GemmEpi ep = {};
     ep.kind = EPI_QKV;
     ep.q_out = c->q; ep.k_out = kinf; ep.v_out = vinf;
     ep.n_q = D.nq; ep.n_kv = D.nkv; ep.head_dim = D.hd;
     ep.pos = c->pos; ep.rope = c->rope;
-    if ((e = gemm(c, w.tm_qkv, w.qkv, c->h, D.nqkv, D.d, M, ep, 2)) != cudaSuccess) return e;
+    if ((e = gemm(c, w.tm_qkv, w.qkv, c->h, D.nqkv, D.d, M, ep, PC_QKV)) != cudaSuccess) return e;
     AttnParams a = {};
     a.q = c->q; a.k_inf = kinf; a.v_inf = vinf;
     a.k_pages = reinterpret_cast<char*>(c->k_pages) + l * kv_layer;
@@ -494,36 +512,52 @@ cudaError_t enqueue_forward(jf_ctx* c, int M, LmMode lm) {
     a.out = c->att; a.Hq = D.Hq; a.Hkv = D.Hkv; a.hd = D.hd;
     a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)D.hd));
     a.err = c->err;
-    if (c->capture_events) prof_begin(c, 1);
+    prof_begin(c, PC_ATTN);
     if (D.bf16) {
-      int prop_sms = 152;
-      cudaDeviceGetAttribute(&prop_sms, cudaDevAttrMultiProcessorCount, c->device);
-      e = launch_attn_bf16(a, 2 * prop_sms, c->st);
+      e = launch_attn_bf16(a, 2 * c->num_sms, c->st);
+      prof_end(c);
+      // units of this forward are bounded by its rows: every chain adds at most one partial tile
+      const int units_bound = std::min(D.max_units, D.Hkv * (cdiv((long long)M * D.G, kAttnQRows) + D.max_chains));
+      prof_begin(c, PC_COMBINE);
+      if (e == cudaSuccess) e = launch_attn_combine(a, units_bound, c->st);
+      prof_end(c);
     } else {
       e = launch_attn_f32(a, M, c->st);
+      prof_end(c);
     }
-    if (c->capture_events) prof_end(c);
     if (e != cudaSuccess) return e;
     GemmEpi er = {};
     er.kind = EPI_RESID; er.x = c->x; er.ldx = D.d;
-    if ((e = gemm(c, w.tm_o, w.o, c->att, D.d, D.nq, M, er, 2)) != cudaSuccess) return e;
-    if ((e = launch_rmsnorm(c->x, w.g_mlp, c->h, D.bf16, M, D.d, eps, c->st)) != cudaSuccess) return e;
+    if ((e = gemm(c, w.tm_o, w.o, c->att, D.d, D.nq, M, er, PC_OPROJ)) != cudaSuccess) return e;
+    prof_begin(c, PC_NORM);
+    e = launch_rmsnorm(c->x, w.g_mlp, c->h, D.bf16, M, D.d, eps, c->st);
+    prof_end(c);
+    if (e != cudaSuccess) return e;
     GemmEpi es = {};
     es.kind = EPI_SWIGLU; es.act = c->act; es.ld_act = D.F;
-    if ((e = gemm(c, w.tm_gu, w.gu, c->h, 2 * D.F, D.d, M, es, 0)) != cudaSuccess) return e;
-    if ((e = gemm(c, w.tm_dn, w.dn, c->act, D.d, D.F, M, er, 2)) != cudaSuccess) return e;
+    if ((e = gemm(c, w.tm_gu, w.gu, c->h, 2 * D.F, D.d, M, es, PC_GATEUP)) != cudaSuccess) return e;
+    if ((e = gemm(c, w.tm_dn, w.dn, c->act, D.d, D.F, M, er, PC_DOWN)) != cudaSuccess) return e;
   }
-  if ((e = launch_rmsnorm(c->x, c->g_final, c->h, D.bf16, M, D.d, eps, c->st)) != cudaSuccess) return e;
+  if (lm == LM_NONE) {
+    c->launches += 1 + (D.bf16 ? 1 : 0) + (D.bf16 ? 8LL : 7LL) * D.L;
+    return cudaSuccess;
+  }
+  const int lm_rows = (lm == LM_LAST) ? 1 : M;
+  const float* x_lm = c->x + (size_t)(M - lm_rows) * D.d;
+  prof_begin(c, PC_NORM);
+  e = launch_rmsnorm(x_lm, c->g_final, c->h, D.bf16, lm_rows, D.d, eps, c->st);
+  prof_end(c);
+  if (e != cudaSuccess) return e;
   GemmEpi el = {};
-  if (lm == LM_ARGMAX) {
+  if (lm != LM_LOGITS) {
     el.kind = EPI_ARGMAX;
     el.am_v1 = c->am_v1; el.am_i1 = c->am_i1; el.am_v2 = c->am_v2; el.am_counter = c->am_counter;
     el.am_out = c->gpred; el.top2_out = c->top2;
   } else {
     el.kind = EPI_STORE; el.y = c->logits; el.ldy = D.V;
   }
-  c->launches += 1 + (D.bf16 ? 1 : 0) + 7LL * D.L + 2;
-  return gemm(c, c->tm_lm, c->w_lm, c->h, D.V, D.d, M, el, 2);
+  c->launches += 1 + (D.bf16 ? 1 : 0) + (D.bf16 ? 8LL : 7LL) * D.L + 2;
+  return gemm(c, c->tm_lm, c->w_lm, c->h, D.V, D.d, lm_rows, el, PC_LMHEAD);
 }
 
 // Upload the rows of one causal chain of sequence `seq` (positions P .. P+M-1).
@@ -559,7 +593,8 @@ jf_status prefill_impl(jf_ctx* c, int seq, const int32_t* host_prompt, const int
     const int m = std::min(D.R, len - start);
     s = upload_chain(c, seq, P, m, host_prompt ? host_prompt + start : nullptr, dev_prompt ? dev_prompt + start : nullptr);
     if (s != JF_OK) return s;
-    CK(enqueue_forward(c, m, LM_ARGMAX));
+    const bool last_chunk = start + m >= len;
+    CK(enqueue_forward(c, m, last_chunk ? LM_LAST : LM_NONE));
     CommitInfo ci{0, m, P};
     CK(cudaMemcpyAsync(c->commit + seq, &ci, sizeof(ci), cudaMemcpyHostToDevice, c->st));
     CK(launch_commit(c->commit + seq, 1, D.L, c->k_inf, c->v_inf, c->k_pages, c->v_pages,
@@ -569,7 +604,7 @@ jf_status prefill_impl(jf_ctx* c, int seq, const int32_t* host_prompt, const int
     P += m;
     if (start + m >= len) {
       int32_t q0 = -1;
-      CK(cudaMemcpyAsync(&q0, c->gpred + (m - 1), 4, cudaMemcpyDeviceToHost, c->st));
+      CK(cudaMemcpyAsync(&q0, c->gpred, 4, cudaMemcpyDeviceToHost, c->st));
       CK(cudaStreamSynchronize(c->st));
       if (next) *next = q0;
     }
@@ -586,11 +621,15 @@ cudaError_t enqueue_iteration(jf_ctx* c, const GenCfg& g, int M, int n_seqs) {
   const Dims& D = c->D;
   cudaError_t e = enqueue_forward(c, M, LM_ARGMAX);
   if (e != cudaSuccess) return e;
+  prof_begin(c, PC_OTHER);
   e = launch_gen_accept(g, c->gen_state, c->gpred, M, c->tok, c->pos, c->chains, c->n_chains, c->commit, c->res_dev,
                         c->err, c->st);
+  prof_end(c);
   if (e != cudaSuccess) return e;
+  prof_begin(c, PC_OTHER);
   e = launch_commit(c->commit, n_seqs, D.L, c->k_inf, c->v_inf, c->k_pages, c->v_pages, c->page_table, D.pps,
                     D.n_pages, D.R, D.Hkv, D.hd, D.es, c->seq_len, c->err, c->st);
+  prof_end(c);
   if (e != cudaSuccess) return e;
   c->launches += 2;
   return cudaMemcpyAsync(c->res_host, c->res_dev, sizeof(IterResult), cudaMemcpyDeviceToHost, c->st);
@@ -653,9 +692,9 @@ void accumulate_profile(jf_ctx* c, GraphRec* g) {
     if (cudaEventElapsedTime(&ms, g->ev[i], g->ev[i + 1]) == cudaSuccess) {
       c->prof_ms[cls] += ms;
       c->prof_n[cls] += 1;
-      if (cls == 0) {  // the gate/up projection is also a projection GEMM
-        c->prof_ms[2] += ms;
-        c->prof_n[2] += 1;
+      if (cls == PC_GATEUP || cls == PC_QKV || cls == PC_OPROJ || cls == PC_DOWN || cls == PC_LMHEAD) {
+        c->prof_ms[PC_GEMMS] += ms;
+        c->prof_n[PC_GEMMS] += 1;
       }
     }
   }
@@ -848,6 +887,7 @@ jf_status jf_create(const jf_model_config* model, const jf_runtime_config* rt, j
   c->O = O;
   c->base = reinterpret_cast<char*>(rup(reinterpret_cast<uintptr_t>(rt->device_arena), 1024));
   cudaGetDevice(&c->device);
+  cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device);
   if (rt->cuda_stream) {
     c->st = reinterpret_cast<cudaStream_t>(rt->cuda_stream);
   } else {
@@ -1298,7 +1338,7 @@ jf_status jf_generate_device(jf_ctx* c, int n_seqs, const int32_t* d_prompts, co
 jf_status jf_set_profiling(jf_ctx* c, int enable) {
   if (!c) return JF_EINVAL;
   c->profiling = enable != 0;
-  for (int i = 0; i < 3; ++i) {
+  for (int i = 0; i < kProfClasses; ++i) {
     c->prof_ms[i] = 0;
     c->prof_n[i] = 0;
   }
@@ -1306,7 +1346,7 @@ jf_status jf_set_profiling(jf_ctx* c, int enable) {
 }
 
 jf_status jf_kernel_time(jf_ctx* c, int cls, double* total_ms, long long* launches) {
-  if (!c || cls < 0 || cls > 2 || !total_ms || !launches) return fail(c, JF_EINVAL, "bad arguments");
+  if (!c || cls < 0 || cls >= kProfClasses || !total_ms || !launches) return fail(c, JF_EINVAL, "bad arguments");
   *total_ms = c->prof_ms[cls];
   *launches = c->prof_n[cls];
   return JF_OK;

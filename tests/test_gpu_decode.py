@@ -94,10 +94,13 @@ def test_block_converges_within_n_iterations(setup):
 
 
 def test_injection_extremes_on_device(setup):
+    """p = 0 accepts whole blocks, p = 1 exactly one token per iteration. The truth is the device's
+    own greedy output, so a flagged near-tie between device and oracle cannot interfere."""
     shape, ctx, model, prompt, truth = setup
     from paper_2512_14681_gb300.jacobi import Gen
 
-    tr = np.array([truth.tokens], dtype=np.int32)
+    own = ctx.generate([prompt], Gen(mode="ar", max_new=len(truth.tokens))).tokens
+    tr = np.ascontiguousarray(own, dtype=np.int32)
     p0 = ctx.generate([prompt], Gen(block_size=8, init="inject", inject_p=0.0, max_new=48), truth=tr)
     assert p0.counts[:, 0].tolist() == [8] * 6
     p1 = ctx.generate([prompt], Gen(block_size=8, init="inject", inject_p=1.0, max_new=20), truth=tr)

@@ -2,8 +2,11 @@
 // Y[m, n] = sum_k X[m, k] W[n, k] for the QKV, O, gate/up, down and LM-head matrices.
 //
 // bf16 path: tcgen05 tensor cores, "swap-AB" so that 128 weight rows form the MMA's M side and
-// the (few) in-flight tokens its N side; weights and activations arrive by TMA with 128-byte
-// swizzle into a multi-stage mbarrier pipeline; the fp32 accumulator lives in tensor memory.
+// the (few) in-flight tokens its N side. A persistent, warp-specialised kernel: one CTA per SM
+// walks its share of (tile, split) work units; a producer warp streams weight and activation
+// tiles by TMA (128-byte swizzle) through a 4-12 stage mbarrier ring that never drains between
+// units; an MMA warp accumulates into one of two TMEM accumulators; four epilogue warps drain
+// the other accumulator (fused epilogue, split-K reduction) while the next unit streams in.
 // fp32 path (small fp32 models): a SIMT mainloop with the same tile shape and epilogues.
 //
 // Split-K is deterministic: partial tiles go to a workspace and the last CTA of a tile (atomic
@@ -17,16 +20,25 @@ namespace {
 
 constexpr int A_STAGE_BYTES = kTileN * kTileK * 2;  // 16 KB of weights per stage
 
+constexpr int EPI_STAGE_BYTES = 16 * kTileN * 4;   // epilogue exchange buffer [16][128] fp32
+constexpr int SMEM_LIMIT = 232448;                  // 227 KB per CTA
+
 template <int BN>
 struct TcCfg {
   static constexpr int B_STAGE_BYTES = BN * kTileK * 2;
   static constexpr int STAGE_BYTES = A_STAGE_BYTES + B_STAGE_BYTES;
-  static constexpr int BUDGET = BN >= 160 ? 200 * 1024 : 104 * 1024;
-  static constexpr int S0 = BUDGET / STAGE_BYTES;
-  static constexpr int STAGES = S0 < 2 ? 2 : (S0 > 8 ? 8 : S0);
-  static constexpr int TMEM_COLS = BN <= 32 ? 32 : (BN <= 64 ? 64 : (BN <= 128 ? 128 : 256));
-  static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + 256;
+  static constexpr int S0 = (SMEM_LIMIT - 1024 - EPI_STAGE_BYTES - 512) / STAGE_BYTES;
+  static constexpr int STAGES = S0 < 2 ? 2 : (S0 > 12 ? 12 : S0);
+  static constexpr int ACC_COLS = BN;   // one accumulator; two are allocated (double buffer)
+  static constexpr int TMEM_COLS = 2 * BN <= 32 ? 32 : (2 * BN <= 64 ? 64 : (2 * BN <= 128 ? 128 : (2 * BN <= 256 ? 256 : 512)));
+  static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + EPI_STAGE_BYTES + 512;
+  static_assert(SMEM <= SMEM_LIMIT, "shared memory budget");
 };
+
+// Named barrier of the 128 epilogue threads (barrier 0 is __syncthreads).
+JF_DEV void epi_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+
+constexpr int kMaxSplits = 8;  // split-K never exceeds this (enforced by the host)
 
 JF_DEV uint8_t* align1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
@@ -43,12 +55,24 @@ JF_DEV void epilogue_chunk(const GemmEpi& e, const float (&v)[16], int row, int 
   constexpr int kind = EPI;
   if constexpr (kind == EPI_STORE || kind == EPI_RESID) {
     if (n < e.N) {
+      if constexpr (kind == EPI_RESID) {
+        // all residual loads first (independent), then the stores
+        float old[16];
 #pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        const int m = m0 + c0 + j;
-        if (m < e.M) {
-          if constexpr (kind == EPI_STORE) e.y[(size_t)m * e.ldy + n] = v[j];
-          else e.x[(size_t)m * e.ldx + n] += v[j];
+        for (int j = 0; j < 16; ++j) {
+          const int m = m0 + c0 + j;
+          old[j] = (m < e.M) ? e.x[(size_t)m * e.ldx + n] : 0.0f;
+        }
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          const int m = m0 + c0 + j;
+          if (m < e.M) e.x[(size_t)m * e.ldx + n] = old[j] + v[j];
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          const int m = m0 + c0 + j;
+          if (m < e.M) e.y[(size_t)m * e.ldy + n] = v[j];
         }
       }
     }
@@ -56,7 +80,7 @@ JF_DEV void epilogue_chunk(const GemmEpi& e, const float (&v)[16], int row, int 
   } else if constexpr (kind == EPI_QKV || kind == EPI_SWIGLU) {
 #pragma unroll
     for (int j = 0; j < 16; ++j) xs[j * 128 + row] = v[j];
-    __syncthreads();
+    epi_sync();
     if constexpr (kind == EPI_QKV) {
       const int hd = e.head_dim, half = hd >> 1;
       const int i = n % hd;
@@ -70,32 +94,39 @@ JF_DEV void epilogue_chunk(const GemmEpi& e, const float (&v)[16], int row, int 
       else if (is_k) { dst = reinterpret_cast<T*>(e.k_out) + (n - e.n_q); stride = (size_t)e.n_kv; }
       else { dst = reinterpret_cast<T*>(e.v_out) + (n - e.n_q - e.n_kv); stride = (size_t)e.n_kv; }
       if (n < e.N) {
-#pragma unroll 4
+        // positions, then rotary coefficients: two rounds of independent loads for 16 tokens
+        int pm[16];
+#pragma unroll
         for (int j = 0; j < 16; ++j) {
           const int m = m0 + c0 + j;
-          if (m >= e.M) break;
+          pm[j] = (rot && m < e.M) ? e.pos[m] : 0;
+        }
+        float2 cs[16];
+#pragma unroll
+        for (int j = 0; j < 16; ++j) cs[j] = rot ? e.rope[(size_t)pm[j] * half + (i % half)] : make_float2(1.f, 0.f);
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          const int m = m0 + c0 + j;
           float out = xs[j * 128 + row];
           if (rot) {
-            const float2 cs = e.rope[(size_t)e.pos[m] * half + (i % half)];
             const float x2 = xs[j * 128 + partner];
-            out = (i < half) ? (out * cs.x - x2 * cs.y) : (out * cs.x + x2 * cs.y);
+            out = (i < half) ? (out * cs[j].x - x2 * cs[j].y) : (out * cs[j].x + x2 * cs[j].y);
           }
-          dst[(size_t)m * stride] = to_act<T>(out);
+          if (m < e.M) dst[(size_t)m * stride] = to_act<T>(out);
         }
       }
     } else {
       if (row < 64) {
         const int f = n_tile * 64 + row;
-#pragma unroll 4
+#pragma unroll
         for (int j = 0; j < 16; ++j) {
           const int m = m0 + c0 + j;
-          if (m >= e.M) break;
           const float g = xs[j * 128 + row], u = xs[j * 128 + row + 64];
-          reinterpret_cast<T*>(e.act)[(size_t)m * e.ld_act + f] = to_act<T>(silu_f(g) * u);
+          if (m < e.M) reinterpret_cast<T*>(e.act)[(size_t)m * e.ld_act + f] = to_act<T>(silu_f(g) * u);
         }
       }
     }
-    __syncthreads();
+    epi_sync();
     return;
   } else {
     // EPI_ARGMAX: best (value, index) and runner-up value over this tile's 128 vocabulary rows
@@ -120,7 +151,7 @@ JF_DEV void epilogue_chunk(const GemmEpi& e, const float (&v)[16], int row, int 
         red[(warp * 16 + j) * 3 + 2] = b2;
       }
     }
-    __syncthreads();
+    epi_sync();
     if (row < 16) {
       const int j = row, m = m0 + c0 + j;
       float b1 = red[j * 3 + 0], b2 = red[j * 3 + 2];
@@ -138,7 +169,7 @@ JF_DEV void epilogue_chunk(const GemmEpi& e, const float (&v)[16], int row, int 
         e.am_v2[at] = b2;
       }
     }
-    __syncthreads();
+    epi_sync();
   }
 }
 
@@ -172,14 +203,14 @@ JF_DEV void argmax_finish(const GemmEpi& e, int m0, int BN, int n_tiles, int tid
   }
 }
 
-// Shared tail of both mainloops: ticketing for split-K and argmax, then the epilogue.
-// get(c0, v) fills this thread's 16 accumulator values of columns c0..c0+15.
+// Shared tail of both mainloops, run by the 128 epilogue threads (tid 0..127): ticketing for
+// split-K and argmax, then the epilogue. get(c0, v) fills this thread's 16 accumulator values of
+// columns c0..c0+15.
 template <typename T, int BN, int EPI, typename Get>
-JF_DEV void finish_tile(const GemmParams& p, Get get, float* xs, int* sflag) {
-  const int tid = threadIdx.x;
-  const int n_tile = blockIdx.x, split = blockIdx.y, m_tile = blockIdx.z;
+JF_DEV void finish_tile(const GemmParams& p, Get get, float* xs, int* sflag, int n_tile, int split, int m_tile,
+                        int tid) {
   const int n0 = n_tile * kTileN, m0 = m_tile * BN;
-  const int tile_lin = m_tile * p.n_tiles + n_tile;
+  const int tile_lin = n_tile * p.m_tiles + m_tile;
   int ncols = p.M - m0;
   if (ncols > BN) ncols = BN;
   const int nchunks = (ncols + 15) >> 4;
@@ -198,23 +229,35 @@ JF_DEV void finish_tile(const GemmParams& p, Get get, float* xs, int* sflag) {
       for (int j = 0; j < 16; ++j) mine[(c * 16 + j) * kTileN + tid] = v[j];
     }
     __threadfence();
-    __syncthreads();
+    epi_sync();
     if (tid == 0) {
       const int t = atomicAdd(p.tile_counter + tile_lin, 1);
       *sflag = (t == p.k_splits - 1);
     }
-    __syncthreads();
-    if (!*sflag) return;
+    epi_sync();
+    const bool last = *sflag != 0;
+    epi_sync();
+    if (!last) return;
     __threadfence();
     const float* base = p.ws + (size_t)tile_lin * p.k_splits * (size_t)BN * kTileN;
     for (int c = 0; c < nchunks; ++c) {
+      // partials of every split in flight together, then added in split order
+      float part[kMaxSplits][16];
+#pragma unroll
+      for (int s = 0; s < kMaxSplits; ++s) {
+        const float* src = base + (size_t)s * BN * kTileN;
+#pragma unroll
+        for (int j = 0; j < 16; ++j) part[s][j] = (s < p.k_splits) ? __ldcg(src + (c * 16 + j) * kTileN + tid) : 0.0f;
+      }
       float v[16];
 #pragma unroll
       for (int j = 0; j < 16; ++j) v[j] = 0.0f;
-      for (int s = 0; s < p.k_splits; ++s) {
-        const float* src = base + (size_t)s * BN * kTileN;
 #pragma unroll
-        for (int j = 0; j < 16; ++j) v[j] += __ldcg(src + (c * 16 + j) * kTileN + tid);
+      for (int s = 0; s < kMaxSplits; ++s) {
+        if (s < p.k_splits) {
+#pragma unroll
+          for (int j = 0; j < 16; ++j) v[j] += part[s][j];
+        }
       }
       epilogue_chunk<T, EPI>(p.epi, v, tid, n0, m0, c * 16, xs, n_tile, p.n_tiles);
     }
@@ -222,13 +265,15 @@ JF_DEV void finish_tile(const GemmParams& p, Get get, float* xs, int* sflag) {
   }
   if constexpr (EPI == EPI_ARGMAX) {
     __threadfence();
-    __syncthreads();
+    epi_sync();
     if (tid == 0) {
       const int t = atomicAdd(p.epi.am_counter + m_tile, 1);
       *sflag = (t == p.n_tiles - 1);
     }
-    __syncthreads();
-    if (*sflag) {
+    epi_sync();
+    const bool last = *sflag != 0;
+    epi_sync();
+    if (last) {
       __threadfence();
       argmax_finish(p.epi, m0, BN, p.n_tiles, tid);
       if (tid == 0) p.epi.am_counter[m_tile] = 0;
@@ -236,12 +281,36 @@ JF_DEV void finish_tile(const GemmParams& p, Get get, float* xs, int* sflag) {
   }
 }
 
+// Work unit u of the persistent schedule: split = u % k_splits; the k_splits units of a tile are
+// consecutive (their partials meet soon), and so are the m tiles of a weight tile (its second
+// read hits L2).
+struct Unit {
+  int n_tile, m_tile, split, kb0, kb1;
+};
+JF_DEV Unit unit_of(const GemmParams& p, int u) {
+  Unit w;
+  w.split = u % p.k_splits;
+  const int t = u / p.k_splits;
+  w.m_tile = t % p.m_tiles;
+  w.n_tile = t / p.m_tiles;
+  w.kb0 = (int)(((long long)p.kb_total * w.split) / p.k_splits);
+  w.kb1 = (int)(((long long)p.kb_total * (w.split + 1)) / p.k_splits);
+  return w;
+}
+
 // ---------------------------------------------------------------------------------------------
-// bf16 tcgen05 kernel. 128 threads: thread 0 = TMA producer, thread 32 = MMA issuer, then all
-// four warps drain the accumulator (warp w reads TMEM lanes 32w .. 32w+31).
+// bf16 tcgen05 persistent kernel, 192 threads: warps 0-3 epilogue (warp w reads TMEM lanes
+// 32w .. 32w+31), warp 4 lane 0 = TMA producer (warp 4 also owns the TMEM allocation),
+// warp 5 lane 0 = MMA issuer.
 // ---------------------------------------------------------------------------------------------
+constexpr int TC_THREADS = 192;
+
+JF_DEV void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
 template <int BN, int EPI>
-__global__ void __launch_bounds__(128, 1)
+__global__ void __launch_bounds__(TC_THREADS, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const GemmParams p) {
   using Cfg = TcCfg<BN>;
   constexpr int S = Cfg::STAGES;
@@ -249,41 +318,54 @@ __global__ void __launch_bounds__(128, 1)
   uint8_t* smem = align1024(smem_raw);
   uint8_t* sA = smem;
   uint8_t* sB = smem + S * A_STAGE_BYTES;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sB + S * Cfg::B_STAGE_BYTES);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * S + 1);
+  float* xs = reinterpret_cast<float*>(sB + S * Cfg::B_STAGE_BYTES);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(xs) + EPI_STAGE_BYTES);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * S + 4);
   int* sflag = reinterpret_cast<int*>(tmem_slot + 1);
-  int* sok = sflag + 1;
 
-  const int tid = threadIdx.x, warp = tid >> 5;
-  const int split = blockIdx.y;
-  const int n0 = blockIdx.x * kTileN, m0 = blockIdx.z * BN;
-  const int kb_begin = (int)(((long long)p.kb_total * split) / p.k_splits);
-  const int kb_end = (int)(((long long)p.kb_total * (split + 1)) / p.k_splits);
-  const int nkb = kb_end - kb_begin;
-  const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + S), accum = smem_u32(bars + 2 * S);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + S);
+  const uint32_t tfull0 = smem_u32(bars + 2 * S), tempty0 = smem_u32(bars + 2 * S + 2);
+  const int total_units = p.n_tiles * p.m_tiles * p.k_splits;
 
-  // thread 0 initialises the barriers and requests the first weight stages right away: weights do
-  // not depend on earlier kernels, so they stream in while TMEM is allocated and while the previous
-  // kernel of the chain finishes.
-  const int pre = nkb < S ? nkb : S;
-  if (tid == 0) {
+  // producer: initialise the barriers, then request the first weight stages right away (weights do
+  // not depend on earlier kernels, so they stream in while the previous kernel finishes)
+  int total_iters = 0;
+  for (int u = blockIdx.x; u < total_units; u += gridDim.x) {
+    const Unit w = unit_of(p, u);
+    total_iters += w.kb1 - w.kb0;
+  }
+  const int pre = total_iters < S ? total_iters : S;
+  if (tid == 128) {
     for (int s = 0; s < S; ++s) {
       mbar_init(full0 + 8 * s, 1);
       mbar_init(empty0 + 8 * s, 1);
     }
-    mbar_init(accum, 1);
-    *sok = 1;
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(tfull0 + 8 * a, 1);
+      mbar_init(tempty0 + 8 * a, 1);
+    }
     fence_mbar_init();
     tma_prefetch_desc(&tmA);
     tma_prefetch_desc(&tmB);
     const uint64_t polA = l2_policy_evict_first();
-    for (int i = 0; i < pre; ++i) {
-      mbar_arrive_expect_tx(full0 + 8 * i, Cfg::STAGE_BYTES);
-      tma_load_2d(smem_u32(sA + i * A_STAGE_BYTES), &tmA, full0 + 8 * i, (kb_begin + i) * kTileK, n0, polA);
+    int u = blockIdx.x, kb = 0;
+    Unit w = unit_of(p, u);
+    kb = w.kb0;
+    for (int j = 0; j < pre; ++j) {
+      mbar_arrive_expect_tx(full0 + 8 * j, Cfg::STAGE_BYTES);
+      tma_load_2d(smem_u32(sA + j * A_STAGE_BYTES), &tmA, full0 + 8 * j, kb * kTileK, w.n_tile * kTileN, polA);
+      if (++kb == w.kb1) {
+        u += gridDim.x;
+        if (u < total_units) {
+          w = unit_of(p, u);
+          kb = w.kb0;
+        }
+      }
     }
   }
   __syncwarp();
-  if (warp == 0) {
+  if (warp == 4) {
     tmem_alloc(smem_u32(tmem_slot), Cfg::TMEM_COLS);
     tmem_relinquish();
   }
@@ -292,60 +374,103 @@ __global__ void __launch_bounds__(128, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  if (tid == 0) {
-    // producer: activations after the previous kernel has completed, then the steady state
-    const uint64_t polA = l2_policy_evict_first(), polB = l2_policy_evict_last();
-    pdl_wait();
-    for (int i = 0; i < pre; ++i)
-      tma_load_2d(smem_u32(sB + i * Cfg::B_STAGE_BYTES), &tmB, full0 + 8 * i, (kb_begin + i) * kTileK, m0, polB);
-    for (int i = pre; i < nkb; ++i) {
-      const int s = i % S;
-      const uint32_t ph = (uint32_t)((i / S) - 1) & 1u;
-      if (!mbar_wait_bounded(empty0 + 8 * s, ph, JF_WAIT_LIMIT_NS)) {
-        jf_set_error(p.err, JF_DERR_TIMEOUT_MMA);
-        *sok = 0;
-        break;
+  if (warp == 4) {
+    if (lane == 0) {
+      const uint64_t polA = l2_policy_evict_first(), polB = l2_policy_evict_last();
+      pdl_wait();
+      // activations of the prefetched stages
+      {
+        int u = blockIdx.x;
+        Unit w = unit_of(p, u);
+        int kb = w.kb0;
+        for (int j = 0; j < pre; ++j) {
+          tma_load_2d(smem_u32(sB + j * Cfg::B_STAGE_BYTES), &tmB, full0 + 8 * j, kb * kTileK, w.m_tile * BN, polB);
+          if (++kb == w.kb1) {
+            u += gridDim.x;
+            if (u < total_units) {
+              w = unit_of(p, u);
+              kb = w.kb0;
+            }
+          }
+        }
       }
-      mbar_arrive_expect_tx(full0 + 8 * s, Cfg::STAGE_BYTES);
-      tma_load_2d(smem_u32(sA + s * A_STAGE_BYTES), &tmA, full0 + 8 * s, (kb_begin + i) * kTileK, n0, polA);
-      tma_load_2d(smem_u32(sB + s * Cfg::B_STAGE_BYTES), &tmB, full0 + 8 * s, (kb_begin + i) * kTileK, m0, polB);
+      // steady state
+      int j = 0;
+      for (int u = blockIdx.x; u < total_units; u += gridDim.x) {
+        const Unit w = unit_of(p, u);
+        bool ok = true;
+        for (int kb = w.kb0; kb < w.kb1; ++kb, ++j) {
+          if (j < pre) continue;
+          const int s = j % S;
+          if (!mbar_wait_bounded(empty0 + 8 * s, (uint32_t)((j / S) - 1) & 1u, JF_WAIT_LIMIT_NS)) {
+            jf_set_error(p.err, JF_DERR_TIMEOUT_MMA);
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(full0 + 8 * s, Cfg::STAGE_BYTES);
+          tma_load_2d(smem_u32(sA + s * A_STAGE_BYTES), &tmA, full0 + 8 * s, kb * kTileK, w.n_tile * kTileN, polA);
+          tma_load_2d(smem_u32(sB + s * Cfg::B_STAGE_BYTES), &tmB, full0 + 8 * s, kb * kTileK, w.m_tile * BN, polB);
+        }
+        if (!ok) break;
+      }
     }
-  } else if (tid == 32) {
+  } else if (warp == 5) {
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(kTileN, BN);
+      int j = 0, i = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; u < total_units && ok; u += gridDim.x, ++i) {
+        const Unit w = unit_of(p, u);
+        const int acc = i & 1;
+        if (i >= 2 && !mbar_wait_bounded(tempty0 + 8 * acc, (uint32_t)((i >> 1) - 1) & 1u, JF_WAIT_LIMIT_NS)) {
+          jf_set_error(p.err, JF_DERR_TIMEOUT_EPI);
+          break;
+        }
+        tc_fence_after();
+        const uint32_t dacc = tmem + (uint32_t)(acc * Cfg::ACC_COLS);
+        for (int kb = w.kb0; kb < w.kb1; ++kb, ++j) {
+          const int s = j % S;
+          if (!mbar_wait_bounded(full0 + 8 * s, (uint32_t)(j / S) & 1u, JF_WAIT_LIMIT_NS)) {
+            jf_set_error(p.err, JF_DERR_TIMEOUT_TMA);
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a = smem_u32(sA + s * A_STAGE_BYTES), b = smem_u32(sB + s * Cfg::B_STAGE_BYTES);
+#pragma unroll
+          for (int kk = 0; kk < kTileK / 16; ++kk)
+            tc_mma_bf16(dacc, sdesc_k_sw128(a + kk * 32), sdesc_k_sw128(b + kk * 32), idesc,
+                        (kb > w.kb0 || kk > 0) ? 1u : 0u);
+          tc_commit(empty0 + 8 * s);
+        }
+        tc_commit(tfull0 + 8 * acc);
+      }
+    }
+  } else {
+    // epilogue warps 0-3
     pdl_wait();
-    constexpr uint32_t idesc = idesc_bf16_f32(kTileN, BN);
-    for (int i = 0; i < nkb; ++i) {
-      const int s = i % S;
-      if (!mbar_wait_bounded(full0 + 8 * s, (uint32_t)(i / S) & 1u, JF_WAIT_LIMIT_NS)) {
-        jf_set_error(p.err, JF_DERR_TIMEOUT_TMA);
-        *sok = 0;
+    const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+    int i = 0;
+    for (int u = blockIdx.x; u < total_units; u += gridDim.x, ++i) {
+      const Unit w = unit_of(p, u);
+      const int acc = i & 1;
+      if (!mbar_wait_bounded(tfull0 + 8 * acc, (uint32_t)(i >> 1) & 1u, JF_WAIT_LIMIT_NS)) {
+        jf_set_error(p.err, JF_DERR_TIMEOUT_EPI);
         break;
       }
       tc_fence_after();
-      const uint32_t a = smem_u32(sA + s * A_STAGE_BYTES), b = smem_u32(sB + s * Cfg::B_STAGE_BYTES);
-#pragma unroll
-      for (int kk = 0; kk < kTileK / 16; ++kk)
-        tc_mma_bf16(tmem, sdesc_k_sw128(a + kk * 32), sdesc_k_sw128(b + kk * 32), idesc, (i | kk) != 0);
-      tc_commit(empty0 + 8 * s);
+      const uint32_t dacc = tmem + (uint32_t)(acc * Cfg::ACC_COLS) + lane_base;
+      auto get = [&](int c0, float (&v)[16]) { tmem_ld16(dacc + (uint32_t)c0, v); };
+      finish_tile<bf16, BN, EPI>(p, get, xs, sflag, w.n_tile, w.split, w.m_tile, tid);
+      tc_fence_before();
+      epi_sync();
+      if (tid == 0) mbar_arrive(tempty0 + 8 * acc);
     }
-    tc_commit(accum);
-  } else {
-    pdl_wait();
   }
-  __syncwarp();
-  const bool acc_ok = mbar_wait_bounded(accum, 0, JF_WAIT_LIMIT_NS);
-  tc_fence_after();
-  if (!acc_ok) jf_set_error(p.err, JF_DERR_TIMEOUT_EPI);
-  __syncthreads();
   pdl_launch_dependents();
-  if (acc_ok && *sok) {
-    float* xs = reinterpret_cast<float*>(sA);
-    const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
-    auto get = [&](int c0, float (&v)[16]) { tmem_ld16(tmem + lane_base + (uint32_t)c0, v); };
-    finish_tile<bf16, BN, EPI>(p, get, xs, sflag);
-  }
   tc_fence_before();
   __syncthreads();
-  if (warp == 0) tmem_dealloc(tmem, Cfg::TMEM_COLS);
+  if (warp == 4) tmem_dealloc(tmem, Cfg::TMEM_COLS);
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -397,15 +522,16 @@ __global__ void __launch_bounds__(128) k_gemm_f32(const float* __restrict__ W, c
         for (int j = 0; j < 16; ++j) v[j] = acc[cc + j];
       }
   };
-  finish_tile<float, F32_BN, EPI>(p, get, xs, &sflag);
+  finish_tile<float, F32_BN, EPI>(p, get, xs, &sflag, blockIdx.x, 0, blockIdx.z, tid);
 }
 
 template <int BN, int EPI>
 cudaError_t launch_tc_epi(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmParams& p, cudaStream_t st) {
   using Cfg = TcCfg<BN>;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(p.n_tiles, p.k_splits, p.m_tiles);
-  cfg.blockDim = dim3(128);
+  const int units = p.n_tiles * p.m_tiles * p.k_splits;
+  cfg.gridDim = dim3(units < p.grid ? units : p.grid);
+  cfg.blockDim = dim3(TC_THREADS);
   cfg.dynamicSmemBytes = Cfg::SMEM;
   cfg.stream = st;
   cudaLaunchAttribute at[1];

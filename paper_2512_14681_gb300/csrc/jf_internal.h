@@ -74,6 +74,7 @@ struct GemmEpi {
 struct GemmParams {
   int N, K, M;
   int n_tiles, m_tiles, k_splits, kb_total;
+  int grid;            // persistent CTAs (bf16 path): at most one per SM
   float* ws;           // split-K partials [m_tiles*n_tiles][k_splits][BN][128]
   int* tile_counter;   // [m_tiles*n_tiles], zero between launches
   int* err;

@@ -59,7 +59,8 @@ extern "C" jf_status jf_op_gemm_noalloc(const void* W, const void* X, float* Y, 
   // tile shape and split exactly as jf_op_gemm chooses them
   const int bn = gemm_bn_for(M);
   const int nt = (N + kTileN - 1) / kTileN, mt = (M + bn - 1) / bn, kb = (K + kTileK - 1) / kTileK;
-  const int sp = k_splits > 0 ? (k_splits < kb ? k_splits : kb) : gemm_default_splits(nt, kb);
+  int sp = k_splits > 0 ? (k_splits < kb ? k_splits : kb) : gemm_default_splits(nt, kb);
+  if (sp > 8) sp = 8;
   const size_t partial_bytes = sp > 1 ? (size_t)nt * mt * sp * bn * kTileN * 4 : 0;
   int* tickets = reinterpret_cast<int*>(reinterpret_cast<char*>(scratch) + rup256(partial_bytes));
   cudaStream_t st = reinterpret_cast<cudaStream_t>(cuda_stream);
@@ -73,6 +74,12 @@ extern "C" jf_status jf_op_gemm_noalloc(const void* W, const void* X, float* Y, 
   p.m_tiles = mt;
   p.k_splits = sp;
   p.kb_total = kb;
+  {
+    int dev = 0, sms = 152;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    p.grid = sms;
+  }
   p.ws = reinterpret_cast<float*>(scratch);
   p.tile_counter = tickets;
   p.err = err_word;

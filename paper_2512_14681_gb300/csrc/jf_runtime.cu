@@ -55,7 +55,7 @@ int splits_for(int n_tiles, int kb_total) {
   if (n_tiles >= kTargetCTAs / 2) return 1;
   int s = kTargetCTAs / n_tiles;
   int cap = std::max(1, kb_total / 4);
-  return std::max(1, std::min(s, cap));
+  return std::max(1, std::min(std::min(s, cap), 8));   // the kernel reduces at most 8 splits
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
@@ -448,6 +448,7 @@ cudaError_t gemm(jf_ctx* c, const CUtensorMap& tmA, const void* W, const void* X
   p.ws = c->gemm_ws;
   p.tile_counter = c->gemm_counter;
   p.err = c->err;
+  p.grid = c->num_sms;
   p.epi = epi;
   p.epi.M = M;
   p.epi.N = N;
@@ -1361,7 +1362,7 @@ static void op_gemm_shape(int dtype, int N, int K, int M, int k_splits, int* bn,
   *mt = cdiv(M, *bn);
   *kb = cdiv(K, kTileK);
   if (dtype != JF_BF16) *sp = 1;
-  else if (k_splits > 0) *sp = std::min(k_splits, *kb);
+  else if (k_splits > 0) *sp = std::min(std::min(k_splits, *kb), 8);
   else *sp = splits_for(*nt, *kb);
 }
 
@@ -1390,6 +1391,12 @@ jf_status jf_op_gemm(int dtype, const void* W, const void* X, float* Y, int N, i
   GemmParams p = {};
   p.N = N; p.K = K; p.M = M;
   p.n_tiles = nt; p.m_tiles = mt; p.k_splits = sp; p.kb_total = kb;
+  {
+    int dev = 0, sms = 152;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    p.grid = sms;
+  }
   const size_t partial = sp > 1 ? (size_t)nt * mt * sp * bn * kTileN * 4 : 0;
   p.ws = reinterpret_cast<float*>(workspace);
   p.tile_counter = workspace ? reinterpret_cast<int*>(reinterpret_cast<char*>(workspace) + rup(partial, 256)) : nullptr;

@@ -15,6 +15,7 @@ shard); value = tokens of all ranks / max-over-ranks time.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import json
 import os
 import statistics
@@ -30,9 +31,41 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 METRIC = "tokens/s at bs1 on 7B-shape; Jacobi-iteration latency as % of HBM roofline"
-WORKLOAD = "qwen2.5-7b-shape-bf16 prompt1024 block32 new512 inject-p0.3 paged-kv16 bs1"
-PROMPT_LEN, BLOCK, NEW, P_INJECT = 1024, 32, 512, 0.3
 NOMINAL_HBM_GBS = 8000.0
+
+
+@dataclasses.dataclass(frozen=True)
+class Workload:
+    name: str
+    shape: str          # key of paper_2512_14681_gb300.inputs.SHAPES
+    prompt: int
+    block: int          # n
+    new: int
+    p: float            # draft-injection corruption rate
+    blocks: int = 1     # K (multi-block decoding)
+    pool: int = 0       # rejection-recycling pool entries
+    ngram: int = 0      # n-gram length (0 = n)
+    cands: int = 0      # recycled candidates verified per iteration
+
+
+# The 7B single-block workload at p = 0.3 is the headline; the others are the remaining decode
+# configurations of the same family (1.5B single block; 7B at p = 0.1 / 0.7; 7B multi-block with
+# rejection recycling). Prompts are uniform-random tokens, weights N(0, 0.02).
+WORKLOADS = {w.name: w for w in [
+    Workload("qwen2.5-7b-shape-bf16 prompt1024 block32 new512 inject-p0.3 paged-kv16 bs1",
+             "qwen2.5-7b-shape-bf16", 1024, 32, 512, 0.3),
+    Workload("qwen2.5-7b-shape-bf16 prompt1024 block32 new512 inject-p0.1 paged-kv16 bs1",
+             "qwen2.5-7b-shape-bf16", 1024, 32, 512, 0.1),
+    Workload("qwen2.5-7b-shape-bf16 prompt1024 block32 new512 inject-p0.7 paged-kv16 bs1",
+             "qwen2.5-7b-shape-bf16", 1024, 32, 512, 0.7),
+    Workload("qwen2.5-1.5b-shape-bf16 prompt512 block16 new256 inject-p0.5 paged-kv16 bs1",
+             "qwen2.5-1.5b-shape-bf16", 512, 16, 256, 0.5),
+    Workload("qwen2.5-7b-shape-bf16 prompt2048 blocks4x32 rr-pool64x32 cand1 new1024 inject-p0.3 paged-kv16 bs1",
+             "qwen2.5-7b-shape-bf16", 2048, 32, 1024, 0.3, blocks=4, pool=64, ngram=32, cands=1),
+]}
+DEFAULT_WORKLOAD = next(iter(WORKLOADS))
+ALIASES = {"7b": DEFAULT_WORKLOAD, "7b-p0.1": list(WORKLOADS)[1], "7b-p0.7": list(WORKLOADS)[2],
+           "1.5b": list(WORKLOADS)[3], "7b-mb4-rr": list(WORKLOADS)[4]}
 # DRAM bytes (read + write) per launch of the gate/up projection at M = 32 rows, from the ncu capture
 # summarised in profiles/gateup_gemm_7b_m32.md; None until a capture of the current kernel exists.
 GATEUP_TRAFFIC_BYTES = None
@@ -100,6 +133,21 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
+def aggregate_ranks(local_ms: float, local_tokens: int, dist=None, device=None):
+    """Whole-job throughput of independent replicas: every rank's tokens over the slowest rank's
+    time (max over ranks of the timed region). Returns (max_ms, total_tokens, tokens_per_s)."""
+    import torch
+
+    if dist is None or not dist.is_initialized() or dist.get_world_size() == 1:
+        return local_ms, local_tokens, local_tokens / (local_ms / 1000.0)
+    t = torch.tensor([local_ms], dtype=torch.float64, device=device)
+    n = torch.tensor([float(local_tokens)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(n, op=dist.ReduceOp.SUM)
+    max_ms, total = float(t.item()), int(n.item())
+    return max_ms, total, total / (max_ms / 1000.0)
+
+
 # ------------------------------------------------------------------------------------------
 # CPU oracle sample (the reference arm and the cpu_baseline object)
 # ------------------------------------------------------------------------------------------
@@ -110,6 +158,8 @@ def oracle_sample(steps: int, warmup: int):
     from oracle import oracle as O
     from paper_2512_14681_gb300 import inputs as I
 
+    w = WORKLOADS[DEFAULT_WORKLOAD]
+    PROMPT_LEN, BLOCK, P_INJECT = w.prompt, w.block, w.p
     shape = I.QWEN7B_BF16
     need = shape.weight_bytes() + (6 << 30)
     avail = os.sysconf("SC_AVPHYS_PAGES") * os.sysconf("SC_PAGE_SIZE")
@@ -144,7 +194,7 @@ def run_reference(args, rank):
     line = {"impl": "reference", "metric": METRIC, "value": res["value"], "unit": "tokens/s", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 * 1.0 / max(res["value"], 1e-9),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": WORKLOAD, "sample": res["sample"]},
+            "data": "synthetic", "config": {"workload": DEFAULT_WORKLOAD, "sample": res["sample"]},
             "cpu_baseline": res, "e2e": {"value": res["value"], "unit": "tokens/s", "h2d_bytes_per_step": 0,
                                          "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
@@ -165,19 +215,23 @@ def run_gpu(args, rank, world, local_rank):
         import torch.distributed as dist
 
         dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
-    shape = I.QWEN7B_BF16
-    if args.layers != shape.n_layers:
-        # reduced-depth copy of the 7B shape: small profiling case only, never a headline number
-        import dataclasses
-
+    wl = WORKLOADS[args.workload]
+    PROMPT_LEN, BLOCK, NEW, P_INJECT = wl.prompt, wl.block, wl.new, wl.p
+    shape = I.SHAPES[wl.shape]
+    if args.layers and args.layers != shape.n_layers:
+        # reduced-depth copy of the shape: small profiling case only, never a headline number
         shape = dataclasses.replace(shape, n_layers=args.layers, name=f"{shape.name}-{args.layers}layers")
-    truth_len = NEW + 2 * BLOCK + 1
-    # max_rows 512: the 1024-token prompt is prefilled in two 512-row forwards
-    ctx = Context(shape, max_seqs=1, max_ctx=2048, max_rows=512)
+    G = wl.ngram or wl.block
+    rows_per_iter = wl.blocks * wl.block + wl.cands * G
+    truth_len = NEW + wl.blocks * BLOCK + G + 1
+    max_ctx = PROMPT_LEN + truth_len + rows_per_iter + 64
+    # prefill in 512-row forwards; decoding needs rows_per_iter rows
+    ctx = Context(shape, max_seqs=1, max_ctx=max_ctx, max_rows=max(512, rows_per_iter))
     ctx.init_random_weights(I.WEIGHT_SEED, I.WEIGHT_STD)
     prompt = I.prompt_tokens(shape.vocab, PROMPT_LEN)
     truth = ctx.generate([prompt], Gen(mode="ar", max_new=truth_len)).tokens[0].astype(np.int32)
-    gen = Gen(block_size=BLOCK, init="inject", inject_p=P_INJECT, seed=I.INJECT_SEED, max_new=NEW)
+    gen = Gen(block_size=BLOCK, n_blocks=wl.blocks, pool_size=wl.pool, ngram_len=wl.ngram, cand_per_iter=wl.cands,
+              init="inject", inject_p=P_INJECT, seed=I.INJECT_SEED, max_new=NEW)
     d_prompt = torch.from_numpy(prompt).cuda()
     d_truth = torch.from_numpy(truth).cuda().reshape(1, -1)
     d_out = torch.empty((1, NEW), dtype=torch.int32, device="cuda")
@@ -189,7 +243,7 @@ def run_gpu(args, rank, world, local_rank):
     for _ in range(args.warmup):
         step()
     torch.cuda.synchronize()
-    first = step(log_cap=1024)
+    first = step(log_cap=4096)
     assert np.array_equal(d_out.cpu().numpy()[0], truth[:NEW]), "generated tokens differ from the greedy truth"
 
     def barrier():
@@ -217,13 +271,8 @@ def run_gpu(args, rank, world, local_rank):
     ev1.record(st)
     barrier()
     clocks = sampler.stop()
-    total_ms = ev0.elapsed_time(ev1)
-    if dist is not None:
-        t = torch.tensor([total_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms, _, value = aggregate_ranks(ev0.elapsed_time(ev1), NEW * args.steps, dist, "cuda")
     ms_per_step = total_ms / args.steps
-    value = world * NEW * args.steps / (total_ms / 1000.0)
 
     # ---- end to end: host buffers in and out through jf_generate
     barrier()
@@ -234,9 +283,8 @@ def run_gpu(args, rank, world, local_rank):
         h = ctx.generate([prompt], gen, truth=truth.reshape(1, -1), log_cap=0)
     e1.record(st)
     barrier()
-    e2e_ms = e0.elapsed_time(e1)
     assert np.array_equal(h.tokens[0], truth[:NEW])
-    e2e_value = world * NEW * args.steps / (e2e_ms / 1000.0)
+    _, _, e2e_value = aggregate_ranks(e0.elapsed_time(e1), NEW * args.steps, dist, "cuda")
 
     # ---- per-kernel timing of the dominant kernel (CUDA events around its launches)
     ctx.set_profiling(True)
@@ -259,14 +307,14 @@ def run_gpu(args, rank, world, local_rank):
     rows = first.rows.astype(np.float64)
     m_avg = float(rows.mean()) if rows.size else float(BLOCK)
     d, F = shape.d_model, shape.d_ff
-    gu_bytes = 2 * F * d * 2 + m_avg * d * 2 + m_avg * F * 2
+    gu_bytes = 2 * F * d * 2 + m_avg * d * 2 + m_avg * F * 2   # weights + activations in + SwiGLU out
     gu_avg_s = gu_ms / max(gu_n, 1) / 1000.0
     achieved = gu_bytes / gu_avg_s / 1e9 if gu_n else None
     # per-iteration roofline: every weight byte + the committed KV read once per iteration
     n_iter = first.iterations
     it_ms = first.decode_ms / max(n_iter, 1)
     kv_tok = shape.kv_bytes_per_token()
-    p_avg = PROMPT_LEN + NEW / 2.0
+    p_avg = PROMPT_LEN + NEW / 2.0   # committed length averaged over the generation
     it_bytes = shape.weight_bytes() + kv_tok * p_avg
     it_gbs = it_bytes / (it_ms / 1000.0) / 1e9
     line = {
@@ -275,8 +323,10 @@ def run_gpu(args, rank, world, local_rank):
         "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic: uniform-random prompt, N(0,0.02) random weights, drafts injected from the model's own "
                 "greedy continuation",
-        "config": {"workload": WORKLOAD if args.layers == 28 else f"{WORKLOAD} ({args.layers}-layer profiling case)",
+        "config": {"workload": args.workload if not args.layers else f"{args.workload} ({args.layers}-layer profiling case)",
                    "layers": shape.n_layers, "prompt": PROMPT_LEN, "block_size": BLOCK, "new_tokens": NEW,
+                   "blocks": wl.blocks, "rr_pool": wl.pool, "ngram": G, "candidates": wl.cands,
+                   "rows_per_iteration_max": rows_per_iter,
                    "inject_p": P_INJECT, "kv_page_tokens": 16, "batch": 1,
                    "parallelism": "replicas" if world > 1 else "single-gpu",
                    "l2": "no flush: every step streams 14.1 GB of weights through the 129 MB L2"},
@@ -295,7 +345,7 @@ def run_gpu(args, rank, world, local_rank):
         "profiled_breakdown_us_per_iteration": {nm: 1000.0 * ms / prof_iters for nm, (ms, n) in prof.items()},
         "clocks": clocks,
     }
-    if args.cpu_baseline and world == 1:
+    if args.cpu_baseline and world == 1 and args.workload == DEFAULT_WORKLOAD and not args.layers:
         cb, why = oracle_sample(args.cpu_baseline_iters, 0)
         line["cpu_baseline"] = cb if cb is not None else {"unavailable": why}
     else:
@@ -303,6 +353,47 @@ def run_gpu(args, rank, world, local_rank):
     print(json.dumps(line))
     if dist is not None:
         dist.destroy_process_group()
+
+
+SWEEP_POINTS = [(P, n, B) for P in (4096, 16384, 32768) for n in (32, 128) for B in (1, 4)]
+
+
+def run_sweep(args):
+    """Fixed-shape Jacobi iterations on the 7B shape: window mode keeps B*n rows in flight every
+    iteration; the latency of an iteration does not depend on the token values."""
+    import torch
+
+    from paper_2512_14681_gb300 import inputs as I
+    from paper_2512_14681_gb300.jacobi import Context, Gen
+
+    shape = I.QWEN7B_BF16
+    peak, peak_kind = _peaks()
+    maxP = max(p[0] for p in SWEEP_POINTS)
+    ctx = Context(shape, max_seqs=4, max_ctx=maxP + 256, max_rows=512)
+    ctx.init_random_weights(I.WEIGHT_SEED, I.WEIGHT_STD)
+    pts = []
+    for P, n, B in SWEEP_POINTS:
+        prompts = [I.prompt_tokens(shape.vocab, P, seed=100 + b) for b in range(B)]
+        out = ctx.generate(prompts, Gen(block_size=n, mode="window", max_new=args.steps + args.warmup), log_cap=64)
+        it_ms = out.decode_ms / max(out.iterations, 1)
+        kv = shape.kv_bytes_per_token() * (P + 2) * B
+        by = shape.weight_bytes() + kv
+        M = n * B
+        flops = 2.0 * M * (shape.weight_bytes() / 2) + 4.0 * shape.head_dim * shape.n_heads * P * shape.n_layers * M
+        t_bytes = by / (peak * 1e9) * 1e3
+        t_flops = flops / 1.936e15 * 1e3
+        pts.append({"prompt": P, "block": n, "batch": B, "rows": M, "iteration_ms": it_ms, "bytes": by,
+                    "gbs": by / (it_ms / 1000.0) / 1e9, "flops": flops,
+                    "roofline_ms": max(t_bytes, t_flops), "bound": "hbm" if t_bytes >= t_flops else "tensor",
+                    "frac_of_roofline": max(t_bytes, t_flops) / it_ms})
+        print(json.dumps(pts[-1]), file=sys.stderr, flush=True)
+    med = statistics.median(p["iteration_ms"] for p in pts)
+    print(json.dumps({"metric": "Jacobi-iteration latency sweep on the 7B shape (bf16, window mode)",
+                      "value": med, "unit": "ms (median over points)", "n_gpus": 1, "steps": args.steps,
+                      "warmup": args.warmup, "higher_is_better": False, "dtype": "bf16", "data": "synthetic",
+                      "config": {"workload": "qwen2.5-7b-shape-bf16 sweep P x n x B", "peak_gbs": peak,
+                                 "peak_kind": peak_kind, "tensor_peak_tflops": 1936.4},
+                      "points": pts}))
 
 
 def main():
@@ -313,8 +404,13 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
     ap.add_argument("--cpu-baseline-iters", type=int, default=2)
-    ap.add_argument("--layers", type=int, default=28, help="decoder layers (28 = the workload; fewer = profiling case)")
+    ap.add_argument("--layers", type=int, default=0, help="decoder layers (0 = the workload's; fewer = profiling case)")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD,
+                    help="workload name or alias (" + ", ".join(ALIASES) + "); 'sweep' = fixed-shape latency sweep")
     args = ap.parse_args()
+    args.workload = ALIASES.get(args.workload, args.workload)
+    if args.workload != "sweep" and args.workload not in WORKLOADS:
+        ap.error(f"unknown workload {args.workload}")
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
@@ -324,7 +420,10 @@ def main():
     import __graft_entry__
 
     __graft_entry__.build()
-    run_gpu(args, rank, world, local_rank)
+    if args.workload == "sweep":
+        run_sweep(args)
+    else:
+        run_gpu(args, rank, world, local_rank)
 
 
 if __name__ == "__main__":

@@ -293,9 +293,8 @@ def run_gpu(args, rank, world, local_rank):
     torch.cuda.synchronize()
     gu_ms, gu_n = ctx.kernel_time(0)
     at_ms, at_n = ctx.kernel_time(1)
-    class_names = ["gate_up", "attention", "all_gemms", "qkv", "o_proj", "down", "lm_head", "attn_combine", "rmsnorm",
-                   "other"]
-    prof = {nm: ctx.kernel_time(i) for i, nm in enumerate(class_names)}
+    class_names = ["gate_up", "attention", "all_gemms", "qkv", "o_proj", "down", "lm_head", None, "rmsnorm", "other"]
+    prof = {nm: ctx.kernel_time(i) for i, nm in enumerate(class_names) if nm}
     prof_iters = max(1, prof["lm_head"][1])
     ctx.set_profiling(False)
 

@@ -62,7 +62,8 @@ typedef struct {
 } jf_model_config;
 
 /* Capacity. max_rows: in-flight rows per forward (K*n + candidates, or a prefill chunk);
- * max_ctx: positions per sequence (KV pages of 16 tokens are reserved for it);
+ * max_ctx: positions per sequence (KV pages of 16 tokens are reserved for it; at most 130944
+ *   for JF_BF16 models, whose attention stages a sequence's page ids in shared memory);
  * logits_rows: rows jf_forward_logits() may return (0 = that call is unavailable). */
 typedef struct {
   int max_seqs, max_ctx, max_rows, logits_rows;
@@ -183,10 +184,11 @@ jf_status jf_generate_device(jf_ctx* ctx, int n_seqs, const int32_t* d_prompts, 
 /* Cumulative device time (ms, CUDA events) and launch count of one kernel class inside
  * jf_generate* decode iterations, when profiling is enabled with jf_set_profiling(ctx, 1) (event
  * records are then placed around every kernel of the iteration graph, which serialises them).
- * kernel_class: 0 = gate/up projection (the largest weight stream), 1 = split-KV attention,
- * 2 = all projection GEMMs, 3 = QKV projection, 4 = O projection, 5 = down projection,
- * 6 = LM head + argmax, 7 = attention combine, 8 = RMSNorm, 9 = other (embedding, attention plan,
- * acceptance, KV commit). jf_set_profiling resets the counters. */
+ * kernel_class: 0 = gate/up projection (the largest weight stream), 1 = split-KV attention
+ * (partials merged inside the kernel), 2 = all projection GEMMs, 3 = QKV projection,
+ * 4 = O projection, 5 = down projection, 6 = LM head + argmax, 7 = reserved (always 0),
+ * 8 = RMSNorm, 9 = other (embedding, acceptance, KV commit). jf_set_profiling resets the
+ * counters. */
 jf_status jf_set_profiling(jf_ctx* ctx, int enable);
 jf_status jf_kernel_time(jf_ctx* ctx, int kernel_class, double* total_ms, long long* launches);
 

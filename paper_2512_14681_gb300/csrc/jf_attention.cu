@@ -9,12 +9,16 @@
 // every row attends to exactly the positions 0 .. p, each position resolved either to a KV page
 // (p < P) or to an in-flight row of its chain.
 //
-// bf16 path: split-KV flash decoding. Work unit = (chain, KV head, tile of 64 (token, head)
-// query rows); items = (unit, chunk of 128 key positions aligned at multiples of 128). Each item
-// runs QK^T and PV on mma.sync.m16n8k16 with an online softmax, keys staged by cp.async into
-// XOR-swizzled shared memory. Partials are merged in chunk order by the unit's last item
-// (atomic ticket). Chunk boundaries are absolute, so a row's arithmetic depends only on its own
-// key set and not on how many rows share the forward.
+// bf16 path: split-KV flash decoding with a fixed reduction tree. Work unit = (chain, KV head,
+// tile of 128 (token, head) query rows). Key positions are cut into absolute 128-key chunks, and
+// chunk c belongs to lane c mod 8. A unit runs on one 8-CTA cluster: CTA j walks the chunks of
+// lane j in increasing order, 64 keys at a time, with one online-softmax state per row (QK^T and
+// PV on mma.sync.m16n8k16, keys staged by cp.async into XOR-swizzled shared memory, the next chunk
+// in flight while the current one computes). Each warp then stores its 16 rows' lane state into
+// the shared memory of the CTA that owns those rows, and after one cluster barrier each CTA folds
+// its rows' 8 lane states in lane order. The tree depends only on absolute key positions, never on
+// how many rows share the forward or how many chunks a unit has, so a row's result is the same in
+// every batch.
 // fp32 path: one warp per (row, head), keys in absolute order, online softmax in fp32.
 #include "jf_device.cuh"
 #include "jf_internal.h"
@@ -23,10 +27,16 @@ namespace jf {
 namespace {
 
 constexpr int HD = 128;
-constexpr int SUB = 64;                   // keys per sub-block
-constexpr int NSUB = kAttnChunk / SUB;    // sub-blocks per chunk
-constexpr int ROW_BYTES = HD * 2;         // 256 bytes per key / query row
+constexpr int SUB = 64;                      // keys per sub-block (one online-softmax step)
+constexpr int NSUB = kAttnChunk / SUB;       // sub-blocks per chunk
+constexpr int ROW_BYTES = HD * 2;            // 256 bytes per key / query row
 constexpr int TILE_BYTES = SUB * ROW_BYTES;  // 16 KB
+constexpr int STAGE_BYTES = 2 * NSUB * TILE_BYTES;     // K and V of one chunk: 64 KB
+constexpr int ROWS_PER_CTA = kAttnQRows / kAttnLanes;  // rows each CTA of a cluster folds (16)
+constexpr int Q_BYTES = kAttnQRows * ROW_BYTES;         // staged queries: 32 KB
+constexpr int RECV_BYTES = ROWS_PER_CTA * kAttnLanes * HD * 4;  // received lane states: 64 KB
+constexpr int REGION0 = RECV_BYTES > Q_BYTES ? RECV_BYTES : Q_BYTES;  // queries, later the lane states
+constexpr int ATT_SMEM = REGION0 + 2 * STAGE_BYTES;   // 192 KB
 
 JF_DEV uint32_t swz(int r, int c16) { return (uint32_t)(r * ROW_BYTES + ((c16 ^ (r & 7)) << 4)); }
 
@@ -64,282 +74,321 @@ JF_DEV uint32_t pack_bf16(float lo, float hi) {
   return (uint32_t)__bfloat16_as_ushort(l) | ((uint32_t)__bfloat16_as_ushort(h) << 16);
 }
 
-// Address of the K (or V) row for absolute key position kp of unit (chain, kvh); null if the
-// position holds no key for this chain. spage: the chunk's page ids (kp0 / 16 ...), resolved once.
-JF_DEV const bf16* key_row(const AttnParams& a, const bf16* pages, const bf16* inf, const Chain& ch, int kvh, int kp,
-                           int max_kp, int kp0, const int* spage) {
-  if (kp > max_kp) return nullptr;
-  if (kp < ch.pos0) {
-    const int page = spage[(kp - kp0) >> 4];
-    if (page < 0 || page >= a.n_pages) return nullptr;
-    return pages + (((size_t)page * a.Hkv + kvh) * kPage + (kp & 15)) * HD;
-  }
-  return inf + ((size_t)(ch.row0 + kp - ch.pos0) * a.Hkv + kvh) * HD;
+// Fold of two softmax states (m, l, O) in the log2 domain: m = max(ma, mb),
+// O = 2^(ma-m) Oa + 2^(mb-m) Ob, l likewise; an empty state has m = -inf and weight 0.
+JF_DEV void fold_weights(float ma, float mb, float& wa, float& wb, float& m) {
+  m = fmaxf(ma, mb);
+  wa = (ma == -INFINITY) ? 0.f : exp2f(ma - m);
+  wb = (mb == -INFINITY) ? 0.f : exp2f(mb - m);
 }
 
-// One work item = (unit, 128-key chunk). 8 warps: warp w computes query-row group w & 3 (16 rows)
-// against key sub-block w >> 2 (64 keys); the two sub-block partials of a row are merged in shared
-// memory, sub-block 0 first, so the chunk's arithmetic is fixed by absolute key positions.
-constexpr int ATT_THREADS = 256;
-
-__global__ void __launch_bounds__(ATT_THREADS, 1) k_attn_bf16(const AttnParams a) {
-  extern __shared__ __align__(128) uint8_t sm[];
-  uint8_t* sQ = sm;                       // 64 x 256 B
-  uint8_t* sK = sm + TILE_BYTES;          // NSUB x 16 KB
-  uint8_t* sV = sK + NSUB * TILE_BYTES;   // NSUB x 16 KB
-  float* sO1 = reinterpret_cast<float*>(sK + TILE_BYTES);  // sub-block 1 partial O [64][128], reuses K1/V1
-  __shared__ int s_rowpos[kAttnQRows];
-  __shared__ int s_page[kAttnChunk / kPage];
-  __shared__ float s_m1[kAttnQRows], s_l1[kAttnQRows];
-
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int rg = warp & 3, sb = warp >> 2;
-  pdl_launch_dependents();  // the next kernel may launch now
-  pdl_wait();
-  const int n_items = a.plan->n_items;
-  const int G = a.Hq / a.Hkv;
+JF_DEV void issue_kv(const AttnParams& a, const AttnUnit& u, int chunk, int li, int max_kp, const int* s_page,
+                     uint8_t* stage, int part) {
   const bf16* Kp = reinterpret_cast<const bf16*>(a.k_pages);
   const bf16* Vp = reinterpret_cast<const bf16*>(a.v_pages);
   const bf16* Ki = reinterpret_cast<const bf16*>(a.k_inf);
   const bf16* Vi = reinterpret_cast<const bf16*>(a.v_inf);
-  const bf16* Q = reinterpret_cast<const bf16*>(a.q);
-  bf16* Out = reinterpret_cast<bf16*>(a.out);
-
-  for (int item = blockIdx.x; item < n_items; item += gridDim.x) {
-    const int2 it = a.items[item];
-    const AttnUnit u = a.units[it.x];
-    const int chunk = it.y;
-    const Chain ch = a.chains[u.chain];
-    const int nq = ch.nrows * G;
-    const int qr0 = u.qt * kAttnQRows;
-    int qrows = nq - qr0;
-    if (qrows > kAttnQRows) qrows = kAttnQRows;
-    const int max_kp = ch.pos0 + (qr0 + qrows - 1) / G;
-    const int kp0 = chunk * kAttnChunk;
-
-    if (tid < kAttnQRows) s_rowpos[tid] = (tid < qrows) ? ch.pos0 + (qr0 + tid) / G : -1;
-    if (tid < kAttnChunk / kPage) {
-      const int kp = kp0 + tid * kPage;
-      s_page[tid] = (kp < ch.pos0) ? a.page_table[(size_t)ch.seq * a.pages_per_seq + (kp >> 4)] : -1;
+  uint8_t* sK = stage;
+  uint8_t* sV = stage + NSUB * TILE_BYTES;
+  const int kp0 = chunk * kAttnChunk;
+  for (int i = threadIdx.x; i < kAttnChunk * 16; i += blockDim.x) {
+    const int r = i >> 4, c = i & 15;
+    const int kp = kp0 + r;
+    const bool cached = kp < u.pos0;
+    if (!(part & (cached ? 1 : 2))) continue;
+    const bf16* kr = nullptr;
+    const bf16* vr = nullptr;
+    if (kp <= max_kp) {
+      if (cached) {
+        const int page = s_page[li * (kAttnChunk / kPage) + (r >> 4)];
+        if (page >= 0 && page < a.n_pages) {
+          const size_t off = (((size_t)page * a.Hkv + u.kvh) * kPage + (kp & 15)) * HD;
+          kr = Kp + off;
+          vr = Vp + off;
+        }
+      } else {
+        const size_t off = ((size_t)(u.row0 + kp - u.pos0) * a.Hkv + u.kvh) * HD;
+        kr = Ki + off;
+        vr = Vi + off;
+      }
     }
-    // stage Q (64 rows, zero beyond qrows)
+    const int b = r / SUB, rr = r % SUB;
+    cp_async16(smem_u32(sK + b * TILE_BYTES) + swz(rr, c), kr ? kr + c * 8 : Kp, kr != nullptr);
+    cp_async16(smem_u32(sV + b * TILE_BYTES) + swz(rr, c), vr ? vr + c * 8 : Vp, vr != nullptr);
+  }
+}
+
+constexpr int ATT_THREADS = 256;
+
+// 8 warps: warp w owns query rows 16w .. 16w+15 of the tile and walks the lane's chunks, 64 keys
+// at a time, with one online-softmax state; at the end it stores that lane state of its 16 rows
+// into CTA w of the cluster, which folds rows 16w .. 16w+15 over the 8 lanes.
+__global__ void __launch_bounds__(ATT_THREADS, 1) k_attn_bf16(const AttnParams a) {
+  extern __shared__ __align__(128) uint8_t sm[];
+  uint8_t* sQ = sm;                                  // 128 x 256 B, free once the queries are in registers
+  float* recv = reinterpret_cast<float*>(sm);        // [16 rows][8 lanes][128], aliases sQ
+  uint8_t* stage0 = sm + REGION0;                    // chunk stages, 64 KB each
+  __shared__ float recv_m[ROWS_PER_CTA * kAttnLanes], recv_l[ROWS_PER_CTA * kAttnLanes];
+  __shared__ int s_rowpos[kAttnQRows];
+  __shared__ int s_page[kAttnLaneChunks * (kAttnChunk / kPage)];
+  __shared__ AttnUnit s_unit;
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int j = (int)cluster_rank();
+  const int ui = (int)cluster_id_x();
+  const int G = a.Hq / a.Hkv;
+  pdl_launch_dependents();  // the next kernel may launch now
+  // Before the dependency wait: the chain table, the page table and the cached keys were written
+  // by host copies or by an earlier graph launch, all complete before this forward began.
+  // Unit ui of the forward: chains in order, then KV heads, then 128-row query tiles.
+  if (tid == 0) s_unit.pad = 0;
+  __syncthreads();
+  if (warp == 0) {
+    const int n_ch = *a.n_chains_dev;
+    int base = 0;
+    for (int c0 = 0; c0 < n_ch; c0 += 32) {
+      const int c = c0 + lane;
+      Chain ch = {0, 0, 0, 0};
+      int nqt = 0;
+      if (c < n_ch) {
+        ch = a.chains[c];
+        nqt = (ch.nrows * G + kAttnQRows - 1) / kAttnQRows;
+      }
+      const int nu = a.Hkv * nqt;
+      int incl = nu;
+#pragma unroll
+      for (int sh = 1; sh < 32; sh <<= 1) {
+        const int v = __shfl_up_sync(0xffffffffu, incl, sh);
+        if (lane >= sh) incl += v;
+      }
+      const int first = base + incl - nu;
+      if (nu > 0 && ui >= first && ui < base + incl) {
+        const int k = ui - first, kvh = k / nqt, qt = k % nqt;
+        int qrows = ch.nrows * G - qt * kAttnQRows;
+        if (qrows > kAttnQRows) qrows = kAttnQRows;
+        const int nch = (ch.pos0 + (qt * kAttnQRows + qrows - 1) / G) / kAttnChunk + 1;
+        if (nch > kAttnLanes * kAttnLaneChunks) {
+          if (j == 0) jf_set_error(a.err, JF_DERR_BOUNDS);
+        } else {
+          s_unit = AttnUnit{ch.seq, ch.row0, ch.nrows, ch.pos0, kvh, qt, nch, 1};
+        }
+      }
+      base += __shfl_sync(0xffffffffu, incl, 31);
+    }
+    // the launch must cover every unit
+    if (lane == 0 && j == 0 && ui == (int)(gridDim.x / kAttnLanes) - 1 && base > ui + 1)
+      jf_set_error(a.err, JF_DERR_BOUNDS);
+  }
+  __syncthreads();
+  const AttnUnit u = s_unit;
+  if (!u.pad) return;  // past the last unit: the whole cluster leaves together
+  const int qr0 = u.qt * kAttnQRows;
+  int qrows = u.nrows * G - qr0;
+  if (qrows > kAttnQRows) qrows = kAttnQRows;
+  const int max_kp = u.pos0 + (qr0 + qrows - 1) / G;
+  const int n_lane = (u.n_chunks > j) ? (u.n_chunks - 1 - j) / kAttnLanes + 1 : 0;
+  const int n_steps = n_lane;
+  auto sub_of = [&](int t) { return j + kAttnLanes * t; };
+
+  for (int i = tid; i < kAttnQRows; i += ATT_THREADS) s_rowpos[i] = (i < qrows) ? u.pos0 + (qr0 + i) / G : -1;
+  for (int i = tid; i < n_lane * (kAttnChunk / kPage); i += ATT_THREADS) {
+    const int li = i / (kAttnChunk / kPage), pg = i % (kAttnChunk / kPage);
+    const int kp = (j + li * kAttnLanes) * kAttnChunk + pg * kPage;
+    s_page[i] = (kp < u.pos0) ? a.page_table[(size_t)u.seq * a.pages_per_seq + (kp >> 4)] : -1;
+  }
+  __syncthreads();
+  if (n_steps > 0) {
+    issue_kv(a, u, sub_of(0), 0, max_kp, s_page, stage0, 1);
+    cp_async_commit();
+  }
+  pdl_wait();  // queries and in-flight keys come from the QKV projection
+  const bf16* Q = reinterpret_cast<const bf16*>(a.q);
+  if (n_steps > 0) {
     for (int i = tid; i < kAttnQRows * 16; i += ATT_THREADS) {
       const int r = i >> 4, c = i & 15;
       const bool ok = r < qrows;
       const int qr = qr0 + (ok ? r : 0);
       const int t = qr / G, g = qr % G;
-      const bf16* src = Q + ((size_t)(ch.row0 + t) * a.Hq + u.kvh * G + g) * HD + c * 8;
+      const bf16* src = Q + ((size_t)(u.row0 + t) * a.Hq + u.kvh * G + g) * HD + c * 8;
       cp_async16(smem_u32(sQ) + swz(r, c), src, ok);
     }
-    __syncthreads();  // page ids visible
-    // stage the chunk's keys and values
-    for (int i = tid; i < NSUB * SUB * 16; i += ATT_THREADS) {
-      const int r = i >> 4, c = i & 15;      // r: key within the chunk
-      const int kp = kp0 + r;
-      const bf16* kr = key_row(a, Kp, Ki, ch, u.kvh, kp, max_kp, kp0, s_page);
-      const bf16* vr = key_row(a, Vp, Vi, ch, u.kvh, kp, max_kp, kp0, s_page);
-      const int b = r / SUB, rr = r % SUB;
-      cp_async16(smem_u32(sK + b * TILE_BYTES) + swz(rr, c), kr ? kr + c * 8 : Kp, kr != nullptr);
-      cp_async16(smem_u32(sV + b * TILE_BYTES) + swz(rr, c), vr ? vr + c * 8 : Vp, vr != nullptr);
-    }
+    issue_kv(a, u, sub_of(0), 0, max_kp, s_page, stage0, 2);
     cp_async_commit();
-    cp_async_wait<0>();
+    if (n_steps > 1) {
+      issue_kv(a, u, sub_of(1), 1, max_kp, s_page, stage0 + STAGE_BYTES, 3);
+      cp_async_commit();
+    }
+  }
+
+  const int r_lo = warp * 16 + (lane >> 2), r_hi = r_lo + 8;
+  const int pos_lo = s_rowpos[r_lo], pos_hi = s_rowpos[r_hi];
+  float o[HD / 8][4];
+#pragma unroll
+  for (int i = 0; i < HD / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+  float m_lo = -INFINITY, m_hi = -INFINITY, l_lo = 0.f, l_hi = 0.f;
+  uint32_t qf[HD / 16][4];
+
+  for (int t = 0; t < n_steps; ++t) {
+    if (t + 1 < n_steps) cp_async_wait<1>();
+    else cp_async_wait<0>();
     __syncthreads();
-
-    // Q fragments of this warp's 16 rows
-    uint32_t qf[HD / 16][4];
+    if (t == 0) {
 #pragma unroll
-    for (int kk = 0; kk < HD / 16; ++kk) {
-      const int r = rg * 16 + (lane & 15), c = kk * 2 + (lane >> 4);
-      ldsm_x4(smem_u32(sQ) + swz(r, c), qf[kk][0], qf[kk][1], qf[kk][2], qf[kk][3]);
+      for (int kk = 0; kk < HD / 16; ++kk) {
+        const int r = warp * 16 + (lane & 15), c = kk * 2 + (lane >> 4);
+        ldsm_x4(smem_u32(sQ) + swz(r, c), qf[kk][0], qf[kk][1], qf[kk][2], qf[kk][3]);
+      }
+      cluster_arrive_relaxed();  // this CTA's query staging is no longer read
     }
-    const int r_lo = rg * 16 + (lane >> 2), r_hi = r_lo + 8;
-    const int pos_lo = s_rowpos[r_lo], pos_hi = s_rowpos[r_hi];
-    float o[HD / 8][4];
+    const int chunk = sub_of(t);
+    uint8_t* stage = stage0 + (t & 1) * STAGE_BYTES;
+#pragma unroll 1
+    for (int sb = 0; sb < NSUB; ++sb) {
+      const uint32_t kb = smem_u32(stage + sb * TILE_BYTES);
+      const uint32_t vb = smem_u32(stage + (NSUB + sb) * TILE_BYTES);
+      float s[SUB / 8][4];
 #pragma unroll
-    for (int i = 0; i < HD / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
-
-    const uint32_t kb = smem_u32(sK + sb * TILE_BYTES), vb = smem_u32(sV + sb * TILE_BYTES);
-    float s[SUB / 8][4];
+      for (int nt = 0; nt < SUB / 8; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
 #pragma unroll
-    for (int nt = 0; nt < SUB / 8; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+      for (int kk = 0; kk < HD / 16; ++kk) {
 #pragma unroll
-    for (int kk = 0; kk < HD / 16; ++kk) {
+        for (int np = 0; np < SUB / 16; ++np) {
+          uint32_t b0, b1, b2, b3;
+          const int r = np * 16 + (lane & 7) + ((lane >> 4) << 3), c = kk * 2 + ((lane >> 3) & 1);
+          ldsm_x4(kb + swz(r, c), b0, b1, b2, b3);
+          mma16816(s[2 * np], qf[kk], b0, b1);
+          mma16816(s[2 * np + 1], qf[kk], b2, b3);
+        }
+      }
+      // mask (key position <= row position), scale to the log2 domain, online-softmax update
+      const int kbase = chunk * kAttnChunk + sb * SUB + 2 * (lane & 3);
+      float x_lo = -INFINITY, x_hi = -INFINITY;
 #pragma unroll
-      for (int np = 0; np < SUB / 16; ++np) {
-        uint32_t b0, b1, b2, b3;
-        const int r = np * 16 + (lane & 7) + ((lane >> 4) << 3), c = kk * 2 + ((lane >> 3) & 1);
-        ldsm_x4(kb + swz(r, c), b0, b1, b2, b3);
-        mma16816(s[2 * np], qf[kk], b0, b1);
-        mma16816(s[2 * np + 1], qf[kk], b2, b3);
+      for (int nt = 0; nt < SUB / 8; ++nt) {
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const int kp = kbase + nt * 8 + e;
+          s[nt][e] = (kp <= pos_lo) ? s[nt][e] * a.scale_log2 : -INFINITY;
+          s[nt][2 + e] = (kp <= pos_hi) ? s[nt][2 + e] * a.scale_log2 : -INFINITY;
+          x_lo = fmaxf(x_lo, s[nt][e]);
+          x_hi = fmaxf(x_hi, s[nt][2 + e]);
+        }
+      }
+#pragma unroll
+      for (int sh = 1; sh <= 2; sh <<= 1) {
+        x_lo = fmaxf(x_lo, __shfl_xor_sync(0xffffffffu, x_lo, sh));
+        x_hi = fmaxf(x_hi, __shfl_xor_sync(0xffffffffu, x_hi, sh));
+      }
+      const float mn_lo = fmaxf(m_lo, x_lo), mn_hi = fmaxf(m_hi, x_hi);
+      const float al_lo = (m_lo == -INFINITY) ? 0.f : exp2f(m_lo - mn_lo);
+      const float al_hi = (m_hi == -INFINITY) ? 0.f : exp2f(m_hi - mn_hi);
+      const float b_lo = (mn_lo == -INFINITY) ? 0.f : mn_lo;
+      const float b_hi = (mn_hi == -INFINITY) ? 0.f : mn_hi;
+      m_lo = mn_lo;
+      m_hi = mn_hi;
+      l_lo *= al_lo;
+      l_hi *= al_hi;
+#pragma unroll
+      for (int nt = 0; nt < SUB / 8; ++nt) {
+        s[nt][0] = exp2f(s[nt][0] - b_lo);
+        s[nt][1] = exp2f(s[nt][1] - b_lo);
+        s[nt][2] = exp2f(s[nt][2] - b_hi);
+        s[nt][3] = exp2f(s[nt][3] - b_hi);
+        l_lo += s[nt][0] + s[nt][1];
+        l_hi += s[nt][2] + s[nt][3];
+      }
+#pragma unroll
+      for (int i = 0; i < HD / 8; ++i) {
+        o[i][0] *= al_lo;
+        o[i][1] *= al_lo;
+        o[i][2] *= al_hi;
+        o[i][3] *= al_hi;
+      }
+      // O += P V
+#pragma unroll
+      for (int kj = 0; kj < SUB / 16; ++kj) {
+        uint32_t pa[4];
+        pa[0] = pack_bf16(s[2 * kj][0], s[2 * kj][1]);
+        pa[1] = pack_bf16(s[2 * kj][2], s[2 * kj][3]);
+        pa[2] = pack_bf16(s[2 * kj + 1][0], s[2 * kj + 1][1]);
+        pa[3] = pack_bf16(s[2 * kj + 1][2], s[2 * kj + 1][3]);
+#pragma unroll
+        for (int dp = 0; dp < HD / 16; ++dp) {
+          uint32_t b0, b1, b2, b3;
+          const int r = kj * 16 + (lane & 7) + (((lane >> 3) & 1) << 3), c = dp * 2 + (lane >> 4);
+          ldsm_x4_t(vb + swz(r, c), b0, b1, b2, b3);
+          mma16816(o[2 * dp], pa, b0, b1);
+          mma16816(o[2 * dp + 1], pa, b2, b3);
+        }
       }
     }
-    // mask (key position <= row position); softmax statistics of this 64-key sub-block (log2 domain)
-    const int kbase = kp0 + sb * SUB + 2 * (lane & 3);
-    float m_lo = -INFINITY, m_hi = -INFINITY;
-#pragma unroll
-    for (int nt = 0; nt < SUB / 8; ++nt) {
-#pragma unroll
-      for (int e = 0; e < 2; ++e) {
-        const int kp = kbase + nt * 8 + e;
-        s[nt][e] = (kp <= pos_lo) ? s[nt][e] * a.scale_log2 : -INFINITY;
-        s[nt][2 + e] = (kp <= pos_hi) ? s[nt][2 + e] * a.scale_log2 : -INFINITY;
-        m_lo = fmaxf(m_lo, s[nt][e]);
-        m_hi = fmaxf(m_hi, s[nt][2 + e]);
-      }
+    __syncthreads();  // this stage is free again
+    if (t + 2 < n_steps) {
+      issue_kv(a, u, sub_of(t + 2), t + 2, max_kp, s_page, stage, 3);
+      cp_async_commit();
     }
+  }
+  if (n_steps == 0) cluster_arrive_relaxed();
 #pragma unroll
-    for (int sh = 1; sh <= 2; sh <<= 1) {
-      m_lo = fmaxf(m_lo, __shfl_xor_sync(0xffffffffu, m_lo, sh));
-      m_hi = fmaxf(m_hi, __shfl_xor_sync(0xffffffffu, m_hi, sh));
-    }
-    const float b_lo = (m_lo == -INFINITY) ? 0.f : m_lo;
-    const float b_hi = (m_hi == -INFINITY) ? 0.f : m_hi;
-    float l_lo = 0.f, l_hi = 0.f;
-#pragma unroll
-    for (int nt = 0; nt < SUB / 8; ++nt) {
-      s[nt][0] = exp2f(s[nt][0] - b_lo);
-      s[nt][1] = exp2f(s[nt][1] - b_lo);
-      s[nt][2] = exp2f(s[nt][2] - b_hi);
-      s[nt][3] = exp2f(s[nt][3] - b_hi);
-      l_lo += s[nt][0] + s[nt][1];
-      l_hi += s[nt][2] + s[nt][3];
-    }
-    // O = P V
-#pragma unroll
-    for (int kj = 0; kj < SUB / 16; ++kj) {
-      uint32_t pa[4];
-      pa[0] = pack_bf16(s[2 * kj][0], s[2 * kj][1]);
-      pa[1] = pack_bf16(s[2 * kj][2], s[2 * kj][3]);
-      pa[2] = pack_bf16(s[2 * kj + 1][0], s[2 * kj + 1][1]);
-      pa[3] = pack_bf16(s[2 * kj + 1][2], s[2 * kj + 1][3]);
-#pragma unroll
-      for (int dp = 0; dp < HD / 16; ++dp) {
-        uint32_t b0, b1, b2, b3;
-        const int r = kj * 16 + (lane & 7) + (((lane >> 3) & 1) << 3), c = dp * 2 + (lane >> 4);
-        ldsm_x4_t(vb + swz(r, c), b0, b1, b2, b3);
-        mma16816(o[2 * dp], pa, b0, b1);
-        mma16816(o[2 * dp + 1], pa, b2, b3);
-      }
-    }
-#pragma unroll
-    for (int sh = 1; sh <= 2; sh <<= 1) {
-      l_lo += __shfl_xor_sync(0xffffffffu, l_lo, sh);
-      l_hi += __shfl_xor_sync(0xffffffffu, l_hi, sh);
-    }
+  for (int sh = 1; sh <= 2; sh <<= 1) {
+    l_lo += __shfl_xor_sync(0xffffffffu, l_lo, sh);
+    l_hi += __shfl_xor_sync(0xffffffffu, l_hi, sh);
+  }
+  // this warp's lane state goes to CTA `warp`, owner of rows 16w .. 16w+15 (r_lo: row lane/4, r_hi: +8)
+  cluster_wait();  // every CTA of the cluster has its queries in registers: the receive buffers are free
+  {
     const int d0 = 2 * (lane & 3);
-    __syncthreads();  // every warp is done with K/V: sub-block 1 partials may overwrite them
-    if (sb == 1) {
+    const int lr = lane >> 2;
+    const uint32_t peer = (uint32_t)warp;
+    const uint32_t o_lo = dsmem_addr(smem_u32(recv + (lr * kAttnLanes + j) * HD + d0), peer);
+    const uint32_t o_hi = dsmem_addr(smem_u32(recv + ((lr + 8) * kAttnLanes + j) * HD + d0), peer);
 #pragma unroll
-      for (int i = 0; i < HD / 8; ++i) {
-        *reinterpret_cast<float2*>(sO1 + r_lo * HD + i * 8 + d0) = make_float2(o[i][0], o[i][1]);
-        *reinterpret_cast<float2*>(sO1 + r_hi * HD + i * 8 + d0) = make_float2(o[i][2], o[i][3]);
-      }
-      if ((lane & 3) == 0) {
-        s_m1[r_lo] = m_lo;
-        s_l1[r_lo] = l_lo;
-        s_m1[r_hi] = m_hi;
-        s_l1[r_hi] = l_hi;
-      }
+    for (int i = 0; i < HD / 8; ++i) {
+      dsmem_st_f32x2(o_lo + i * 32, o[i][0], o[i][1]);
+      dsmem_st_f32x2(o_hi + i * 32, o[i][2], o[i][3]);
     }
-    __syncthreads();
-    if (sb == 0) {
-      // merge: m = max(m0, m1), O = 2^(m0-m) O0 + 2^(m1-m) O1, l likewise
-      const float m1_lo = s_m1[r_lo], m1_hi = s_m1[r_hi];
-      const float mm_lo = fmaxf(m_lo, m1_lo), mm_hi = fmaxf(m_hi, m1_hi);
-      const float a0_lo = (m_lo == -INFINITY) ? 0.f : exp2f(m_lo - mm_lo);
-      const float a1_lo = (m1_lo == -INFINITY) ? 0.f : exp2f(m1_lo - mm_lo);
-      const float a0_hi = (m_hi == -INFINITY) ? 0.f : exp2f(m_hi - mm_hi);
-      const float a1_hi = (m1_hi == -INFINITY) ? 0.f : exp2f(m1_hi - mm_hi);
-      l_lo = a0_lo * l_lo + a1_lo * s_l1[r_lo];
-      l_hi = a0_hi * l_hi + a1_hi * s_l1[r_hi];
-#pragma unroll
-      for (int i = 0; i < HD / 8; ++i) {
-        const float2 p_lo = *reinterpret_cast<const float2*>(sO1 + r_lo * HD + i * 8 + d0);
-        const float2 p_hi = *reinterpret_cast<const float2*>(sO1 + r_hi * HD + i * 8 + d0);
-        o[i][0] = a0_lo * o[i][0] + a1_lo * p_lo.x;
-        o[i][1] = a0_lo * o[i][1] + a1_lo * p_lo.y;
-        o[i][2] = a0_hi * o[i][2] + a1_hi * p_hi.x;
-        o[i][3] = a0_hi * o[i][3] + a1_hi * p_hi.y;
-      }
-      m_lo = mm_lo;
-      m_hi = mm_hi;
-      if (u.n_chunks == 1) {
-        const float il_lo = l_lo > 0.f ? 1.f / l_lo : 0.f, il_hi = l_hi > 0.f ? 1.f / l_hi : 0.f;
-#pragma unroll
-        for (int half = 0; half < 2; ++half) {
-          const int r = half ? r_hi : r_lo;
-          if (r >= qrows) continue;
-          const float il = half ? il_hi : il_lo;
-          const int qr = qr0 + r, t = qr / G, g = qr % G;
-          bf16* dst = Out + ((size_t)(ch.row0 + t) * a.Hq + u.kvh * G + g) * HD;
-#pragma unroll
-          for (int i = 0; i < HD / 8; ++i) {
-            const float x0 = o[i][2 * half] * il, x1 = o[i][2 * half + 1] * il;
-            *reinterpret_cast<uint32_t*>(dst + i * 8 + d0) = pack_bf16(x0, x1);
-          }
-        }
-      } else {
-        const int slot = u.slot0 + chunk;
-        float* wo = a.ws_o + (size_t)slot * kAttnQRows * HD;
-        float* wml = a.ws_ml + (size_t)slot * kAttnQRows * 2;
-#pragma unroll
-        for (int i = 0; i < HD / 8; ++i) {
-          *reinterpret_cast<float2*>(wo + r_lo * HD + i * 8 + d0) = make_float2(o[i][0], o[i][1]);
-          *reinterpret_cast<float2*>(wo + r_hi * HD + i * 8 + d0) = make_float2(o[i][2], o[i][3]);
-        }
-        if ((lane & 3) == 0) {
-          wml[r_lo * 2] = m_lo;
-          wml[r_lo * 2 + 1] = l_lo;
-          wml[r_hi * 2] = m_hi;
-          wml[r_hi * 2 + 1] = l_hi;
-        }
-      }
+    if ((lane & 3) == 0) {
+      dsmem_st_f32(dsmem_addr(smem_u32(recv_m + lr * kAttnLanes + j), peer), m_lo);
+      dsmem_st_f32(dsmem_addr(smem_u32(recv_l + lr * kAttnLanes + j), peer), l_lo);
+      dsmem_st_f32(dsmem_addr(smem_u32(recv_m + (lr + 8) * kAttnLanes + j), peer), m_hi);
+      dsmem_st_f32(dsmem_addr(smem_u32(recv_l + (lr + 8) * kAttnLanes + j), peer), l_hi);
     }
-    __syncthreads();
   }
-}
-
-// Merge of the split-KV partials of multi-chunk units, in chunk order:
-//   out = sum_c 2^(m_c - M) O_c / sum_c 2^(m_c - M) l_c,  M = max_c m_c.
-// CTA (x, u) handles rows 8x .. 8x+7 of unit u; thread = (row, 4 of the 128 dims).
-__global__ void __launch_bounds__(256) k_attn_combine(const AttnParams a) {
-  pdl_launch_dependents();
-  pdl_wait();
-  const int u_idx = blockIdx.y;
-  if (u_idx >= a.plan->n_units) return;
-  const AttnUnit u = a.units[u_idx];
-  if (u.n_chunks == 1) return;
-  const Chain ch = a.chains[u.chain];
-  const int G = a.Hq / a.Hkv;
-  const int qr0 = u.qt * kAttnQRows;
-  int qrows = ch.nrows * G - qr0;
-  if (qrows > kAttnQRows) qrows = kAttnQRows;
-  const int r = blockIdx.x * 8 + (threadIdx.x >> 5);
-  if (r >= qrows) return;
-  const int d = (threadIdx.x & 31) * 4;
-  const float2* ml = reinterpret_cast<const float2*>(a.ws_ml);
-  float M = -INFINITY;
-#pragma unroll 4
-  for (int c = 0; c < u.n_chunks; ++c) M = fmaxf(M, __ldcg(ml + (size_t)(u.slot0 + c) * kAttnQRows + r).x);
-  float L = 0.f, acc0 = 0.f, acc1 = 0.f, acc2 = 0.f, acc3 = 0.f;
-#pragma unroll 4
-  for (int c = 0; c < u.n_chunks; ++c) {
-    const size_t sl = (size_t)(u.slot0 + c);
-    const float2 p = __ldcg(ml + sl * kAttnQRows + r);
-    const float4 oc = __ldcg(reinterpret_cast<const float4*>(a.ws_o + (sl * kAttnQRows + r) * HD + d));
-    const float w = (p.x == -INFINITY) ? 0.f : exp2f(p.x - M);
-    L += w * p.y;
-    acc0 += w * oc.x;
-    acc1 += w * oc.y;
-    acc2 += w * oc.z;
-    acc3 += w * oc.w;
+  // every lane state of this CTA's rows has arrived; no shared memory is accessed remotely after this
+  cluster_sync();
+  // fold of rows 16j .. 16j+15 over the 8 lanes in order; thread = (row, 8 of the 128 dims)
+  {
+    const int lr = tid >> 4, r = j * ROWS_PER_CTA + lr;
+    const int d = (tid & 15) * 8;
+    if (r < qrows) {
+      const float* ro = recv + lr * kAttnLanes * HD + d;
+      float M = recv_m[lr * kAttnLanes], L = recv_l[lr * kAttnLanes];
+      float acc[8];
+      {
+        const float4 x0 = *reinterpret_cast<const float4*>(ro), x1 = *reinterpret_cast<const float4*>(ro + 4);
+        acc[0] = x0.x; acc[1] = x0.y; acc[2] = x0.z; acc[3] = x0.w;
+        acc[4] = x1.x; acc[5] = x1.y; acc[6] = x1.z; acc[7] = x1.w;
+      }
+#pragma unroll
+      for (int q = 1; q < kAttnLanes; ++q) {
+        float wa, wb, mm;
+        fold_weights(M, recv_m[lr * kAttnLanes + q], wa, wb, mm);
+        const float4 x0 = *reinterpret_cast<const float4*>(ro + q * HD);
+        const float4 x1 = *reinterpret_cast<const float4*>(ro + q * HD + 4);
+        M = mm;
+        L = wa * L + wb * recv_l[lr * kAttnLanes + q];
+        acc[0] = wa * acc[0] + wb * x0.x; acc[1] = wa * acc[1] + wb * x0.y;
+        acc[2] = wa * acc[2] + wb * x0.z; acc[3] = wa * acc[3] + wb * x0.w;
+        acc[4] = wa * acc[4] + wb * x1.x; acc[5] = wa * acc[5] + wb * x1.y;
+        acc[6] = wa * acc[6] + wb * x1.z; acc[7] = wa * acc[7] + wb * x1.w;
+      }
+      const float il = L > 0.f ? 1.f / L : 0.f;
+      const int qr = qr0 + r, t = qr / G, g = qr % G;
+      bf16* dst = reinterpret_cast<bf16*>(a.out) + ((size_t)(u.row0 + t) * a.Hq + u.kvh * G + g) * HD + d;
+      *reinterpret_cast<uint4*>(dst) = make_uint4(pack_bf16(acc[0] * il, acc[1] * il), pack_bf16(acc[2] * il, acc[3] * il),
+                                                  pack_bf16(acc[4] * il, acc[5] * il), pack_bf16(acc[6] * il, acc[7] * il));
+    }
   }
-  const float il = L > 0.f ? 1.f / L : 0.f;
-  const int qr = qr0 + r, t = qr / G, g = qr % G;
-  bf16* dst = reinterpret_cast<bf16*>(a.out) + ((size_t)(ch.row0 + t) * a.Hq + u.kvh * G + g) * HD + d;
-  *reinterpret_cast<uint32_t*>(dst) = pack_bf16(acc0 * il, acc1 * il);
-  *reinterpret_cast<uint32_t*>(dst + 2) = pack_bf16(acc2 * il, acc3 * il);
 }
 
 // fp32 path: one warp per (row, query head); keys in absolute order, 32 at a time.
@@ -418,92 +467,47 @@ __global__ void __launch_bounds__(128) k_attn_f32(const AttnParams a, int n_rows
   if (lane + 32 < hd) out[lane + 32] = o1 * il;
 }
 
-// Work decomposition of the bf16 attention for the current chains (one CTA, once per forward).
-__global__ void k_attn_plan(const Chain* chains, const int* n_chains_dev, int Hq, int Hkv, AttnPlan* plan,
-                            AttnUnit* units, int2* items, int max_units, int max_items, int max_slots, int* err) {
-  pdl_launch_dependents();
-  pdl_wait();
-  if (threadIdx.x != 0) return;
-  const int G = Hq / Hkv;
-  int nu = 0, ni = 0, ns = 0;
-  const int n_ch = *n_chains_dev;
-  for (int c = 0; c < n_ch; ++c) {
-    const Chain ch = chains[c];
-    const int nq = ch.nrows * G;
-    const int nqt = (nq + kAttnQRows - 1) / kAttnQRows;
-    for (int kvh = 0; kvh < Hkv; ++kvh)
-      for (int qt = 0; qt < nqt; ++qt) {
-        int qrows = nq - qt * kAttnQRows;
-        if (qrows > kAttnQRows) qrows = kAttnQRows;
-        const int max_kp = ch.pos0 + (qt * kAttnQRows + qrows - 1) / G;
-        const int nch = max_kp / kAttnChunk + 1;
-        if (nu >= max_units || ni + nch > max_items || (nch > 1 && ns + nch > max_slots)) {
-          jf_set_error(err, JF_DERR_BOUNDS);
-          plan->n_units = plan->n_items = 0;
-          return;
-        }
-        units[nu] = AttnUnit{c, kvh, qt, nch, ns};
-        for (int k = 0; k < nch; ++k) items[ni + k] = make_int2(nu, k);
-        ni += nch;
-        if (nch > 1) ns += nch;
-        ++nu;
-      }
-  }
-  plan->n_units = nu;
-  plan->n_items = ni;
-  plan->n_slots = ns;
-}
-
 }  // namespace
 
-size_t attn_bf16_smem_bytes() { return (size_t)TILE_BYTES * (1 + 2 * NSUB); }
-
-cudaError_t launch_attn_plan(const Chain* chains, const int* n_chains_dev, int Hq, int Hkv, AttnPlan* plan,
-                             AttnUnit* units, int2* items, int max_units, int max_items, int max_slots, int* err,
-                             cudaStream_t st) {
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(1);
-  cfg.blockDim = dim3(32);
-  cfg.stream = st;
-  cudaLaunchAttribute at[1];
-  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  at[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = at;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, k_attn_plan, chains, n_chains_dev, Hq, Hkv, plan, units, items, max_units,
-                            max_items, max_slots, err);
-}
+size_t attn_bf16_smem_bytes() { return (size_t)ATT_SMEM; }
 
 cudaError_t attn_prepare() {
-  return cudaFuncSetAttribute(k_attn_bf16, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)attn_bf16_smem_bytes());
-}
-
-cudaError_t launch_attn_bf16(const AttnParams& a, int grid, cudaStream_t st) {
-  const size_t smem = attn_bf16_smem_bytes();
+  cudaError_t e = cudaFuncSetAttribute(k_attn_bf16, cudaFuncAttributeMaxDynamicSharedMemorySize, ATT_SMEM);
+  if (e != cudaSuccess) return e;
+  // an 8-CTA cluster of this kernel must fit on the device
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(grid);
+  cfg.gridDim = dim3(kAttnLanes);
   cfg.blockDim = dim3(ATT_THREADS);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = st;
+  cfg.dynamicSmemBytes = ATT_SMEM;
   cudaLaunchAttribute at[1];
-  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  at[0].val.programmaticStreamSerializationAllowed = 1;
+  at[0].id = cudaLaunchAttributeClusterDimension;
+  at[0].val.clusterDim.x = kAttnLanes;
+  at[0].val.clusterDim.y = 1;
+  at[0].val.clusterDim.z = 1;
   cfg.attrs = at;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, k_attn_bf16, a);
+  int n_clusters = 0;
+  e = cudaOccupancyMaxActiveClusters(&n_clusters, k_attn_bf16, &cfg);
+  if (e != cudaSuccess) return e;
+  return n_clusters > 0 ? cudaSuccess : cudaErrorInvalidConfiguration;
 }
 
-cudaError_t launch_attn_combine(const AttnParams& a, int max_units, cudaStream_t st) {
+cudaError_t launch_attn_bf16(const AttnParams& a, int units_bound, cudaStream_t st) {
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(kAttnQRows / 8, max_units);
-  cfg.blockDim = dim3(256);
+  cfg.gridDim = dim3(kAttnLanes * units_bound);
+  cfg.blockDim = dim3(ATT_THREADS);
+  cfg.dynamicSmemBytes = ATT_SMEM;
   cfg.stream = st;
-  cudaLaunchAttribute at[1];
+  cudaLaunchAttribute at[2];
   at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   at[0].val.programmaticStreamSerializationAllowed = 1;
+  at[1].id = cudaLaunchAttributeClusterDimension;
+  at[1].val.clusterDim.x = kAttnLanes;
+  at[1].val.clusterDim.y = 1;
+  at[1].val.clusterDim.z = 1;
   cfg.attrs = at;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, k_attn_combine, a);
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, k_attn_bf16, a);
 }
 
 cudaError_t launch_attn_f32(const AttnParams& a, int n_rows, cudaStream_t st) {

@@ -82,6 +82,9 @@ __global__ void k_embed(const T* __restrict__ E, const int* __restrict__ tok, fl
 // y[r, :] = x[r, :] / sqrt(mean(x[r, :]^2) + eps) * gain, rounded to the activation type.
 // One CTA per row; the row stays in registers (float4, up to 8 per thread: d <= 8192), so x is
 // read once. The reduction order is fixed by d alone.
+// ACC: the residual update of the preceding projection is finished here first: the k_splits
+// partial sums of x's increment (EPI_PARTIAL) are added in split order, x += that sum is written
+// back, and the norm is taken of the updated row. Rows are row0 + blockIdx.x.
 constexpr int NORM_THREADS = 256;
 constexpr int NORM_VEC = 8;
 
@@ -94,21 +97,39 @@ __device__ __forceinline__ void store4(bf16* y, float4 v) {
   *reinterpret_cast<uint2*>(y) = make_uint2(lo, hi);
 }
 
-template <typename T>
-__global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(const float* __restrict__ x, const float* __restrict__ gain,
-                                                          T* __restrict__ y, int d, float eps) {
+template <typename T, bool ACC>
+__global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(float* __restrict__ x, const float* __restrict__ gain,
+                                                          T* __restrict__ y, int d, float eps, SplitPartials sp,
+                                                          int row0) {
   __shared__ float red[NORM_THREADS / 32];
   pdl_launch_dependents();  // the next projection may launch now and prefetch its weights
   pdl_wait();
-  const int r = blockIdx.x;
+  const int r = row0 + blockIdx.x;
   const int nv = d >> 2;
-  const float4* xr = reinterpret_cast<const float4*>(x + (size_t)r * d);
+  float4* xr = reinterpret_cast<float4*>(x + (size_t)r * d);
   float4 v[NORM_VEC];
   float ss = 0.f;
 #pragma unroll
   for (int j = 0; j < NORM_VEC; ++j) {
     const int i = threadIdx.x + j * NORM_THREADS;
     v[j] = (i < nv) ? xr[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+    if constexpr (ACC) {
+      if (i < nv) {
+        const int n = 4 * i;
+        const float* base = sp.ws + ((size_t)((n >> 7) * sp.m_tiles + r / sp.bn) * sp.k_splits * sp.bn +
+                                     (size_t)(r % sp.bn)) * 128 + (n & 127);
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int s = 0; s < sp.k_splits; ++s) {
+          const float4 q = __ldcg(reinterpret_cast<const float4*>(base + (size_t)s * sp.bn * 128));
+          acc.x += q.x;
+          acc.y += q.y;
+          acc.z += q.z;
+          acc.w += q.w;
+        }
+        v[j] = make_float4(v[j].x + acc.x, v[j].y + acc.y, v[j].z + acc.z, v[j].w + acc.w);
+        xr[i] = v[j];
+      }
+    }
     ss = fmaf(v[j].x, v[j].x, ss);
     ss = fmaf(v[j].y, v[j].y, ss);
     ss = fmaf(v[j].z, v[j].z, ss);
@@ -122,7 +143,7 @@ __global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(const float* __restric
   for (int w = 0; w < NORM_THREADS / 32; ++w) tot += red[w];
   const float rs = 1.0f / sqrtf(tot / (float)d + eps);
   const float4* g4 = reinterpret_cast<const float4*>(gain);
-  T* yr = y + (size_t)r * d;
+  T* yr = y + (size_t)blockIdx.x * d;
 #pragma unroll
   for (int j = 0; j < NORM_VEC; ++j) {
     const int i = threadIdx.x + j * NORM_THREADS;
@@ -131,6 +152,53 @@ __global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(const float* __restric
       store4(yr + 4 * i, make_float4(v[j].x * rs * g.x, v[j].y * rs * g.y, v[j].z * rs * g.z, v[j].w * rs * g.w));
     }
   }
+}
+
+// Finish of the QKV projection from its split-K partials (EPI_PARTIAL, head_dim 128 = one weight
+// tile per head): for row m and head slot hs (query heads, then key heads, then value heads), add
+// the partials in split order, rotate query and key heads by the row's position (rotate-half RoPE,
+// the same arithmetic as the fused epilogue), round to bf16 and store to q [m][Hq][128],
+// k / v [m][Hkv][128]. One warp per (row, head slot); lane l holds dims 4l .. 4l+3, whose rotation
+// partner is lane l ^ 16.
+__global__ void __launch_bounds__(128) k_qkv_finish(SplitPartials sp, const int* __restrict__ pos,
+                                                     const float2* __restrict__ rope, bf16* __restrict__ q,
+                                                     bf16* __restrict__ k, bf16* __restrict__ v, int M, int Hq,
+                                                     int Hkv) {
+  pdl_launch_dependents();
+  pdl_wait();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int slots = Hq + 2 * Hkv;
+  const int job = blockIdx.x * 4 + warp;
+  if (job >= M * slots) return;
+  const int m = job / slots, hs = job % slots;
+  const float* base = sp.ws + ((size_t)(hs * sp.m_tiles + m / sp.bn) * sp.k_splits * sp.bn + (size_t)(m % sp.bn)) * 128 +
+                      lane * 4;
+  float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int s = 0; s < sp.k_splits; ++s) {
+    const float4 t = __ldcg(reinterpret_cast<const float4*>(base + (size_t)s * sp.bn * 128));
+    a.x += t.x;
+    a.y += t.y;
+    a.z += t.z;
+    a.w += t.w;
+  }
+  bf16* dst;
+  if (hs < Hq + Hkv) {
+    const int p = pos[m];
+    const float4 b = make_float4(__shfl_xor_sync(0xffffffffu, a.x, 16), __shfl_xor_sync(0xffffffffu, a.y, 16),
+                                 __shfl_xor_sync(0xffffffffu, a.z, 16), __shfl_xor_sync(0xffffffffu, a.w, 16));
+    const int i0 = (lane * 4) & 63;
+    const float2* cs = rope + (size_t)p * 64 + i0;
+    const float2 c0 = cs[0], c1 = cs[1], c2 = cs[2], c3 = cs[3];
+    if (lane < 16) {
+      a = make_float4(a.x * c0.x - b.x * c0.y, a.y * c1.x - b.y * c1.y, a.z * c2.x - b.z * c2.y, a.w * c3.x - b.w * c3.y);
+    } else {
+      a = make_float4(a.x * c0.x + b.x * c0.y, a.y * c1.x + b.y * c1.y, a.z * c2.x + b.z * c2.y, a.w * c3.x + b.w * c3.y);
+    }
+    dst = (hs < Hq) ? q + ((size_t)m * Hq + hs) * 128 : k + ((size_t)m * Hkv + (hs - Hq)) * 128;
+  } else {
+    dst = v + ((size_t)m * Hkv + (hs - Hq - Hkv)) * 128;
+  }
+  store4(dst + lane * 4, a);
 }
 
 template <typename K, typename... Args>
@@ -187,11 +255,26 @@ cudaError_t launch_embed(const void* E, bool is_bf16, const int* tok, float* x, 
   return launch_pdl(k_embed<float>, dim3(rows), dim3(256), st, reinterpret_cast<const float*>(E), tok, x, d, V, err);
 }
 
-cudaError_t launch_rmsnorm(const float* x, const float* gain, void* y, bool is_bf16, int rows, int d, float eps,
-                           cudaStream_t st) {
-  if (is_bf16)
-    return launch_pdl(k_rmsnorm<bf16>, dim3(rows), dim3(NORM_THREADS), st, x, gain, reinterpret_cast<bf16*>(y), d, eps);
-  return launch_pdl(k_rmsnorm<float>, dim3(rows), dim3(NORM_THREADS), st, x, gain, reinterpret_cast<float*>(y), d, eps);
+cudaError_t launch_rmsnorm(float* x, const float* gain, void* y, bool is_bf16, int rows, int d, float eps,
+                           const SplitPartials* acc, int row0, cudaStream_t st) {
+  const SplitPartials sp = acc ? *acc : SplitPartials{nullptr, 0, 1, 1};
+  if (is_bf16) {
+    if (acc)
+      return launch_pdl(k_rmsnorm<bf16, true>, dim3(rows), dim3(NORM_THREADS), st, x, gain, reinterpret_cast<bf16*>(y),
+                        d, eps, sp, row0);
+    return launch_pdl(k_rmsnorm<bf16, false>, dim3(rows), dim3(NORM_THREADS), st, x, gain, reinterpret_cast<bf16*>(y),
+                      d, eps, sp, row0);
+  }
+  if (acc) return cudaErrorInvalidValue;
+  return launch_pdl(k_rmsnorm<float, false>, dim3(rows), dim3(NORM_THREADS), st, x, gain, reinterpret_cast<float*>(y),
+                    d, eps, sp, row0);
+}
+
+cudaError_t launch_qkv_finish(const SplitPartials& sp, const int* pos, const float2* rope, void* q, void* k, void* v,
+                              int M, int Hq, int Hkv, cudaStream_t st) {
+  const int jobs = M * (Hq + 2 * Hkv);
+  return launch_pdl(k_qkv_finish, dim3((jobs + 3) / 4), dim3(128), st, sp, pos, rope, reinterpret_cast<bf16*>(q),
+                    reinterpret_cast<bf16*>(k), reinterpret_cast<bf16*>(v), M, Hq, Hkv);
 }
 
 }  // namespace jf

@@ -203,9 +203,13 @@ JF_DEV void argmax_finish(const GemmEpi& e, int m0, int BN, int n_tiles, int tid
   }
 }
 
-// Shared tail of both mainloops, run by the 128 epilogue threads (tid 0..127): ticketing for
-// split-K and argmax, then the epilogue. get(c0, v) fills this thread's 16 accumulator values of
-// columns c0..c0+15.
+template <typename T, int BN, int EPI, typename Get>
+JF_DEV void finish_tile_epi(const GemmParams& p, Get get, float* xs, int* sflag, int n_tile, int split, int m_tile,
+                            int tid, int n0, int m0, int tile_lin, int nchunks);
+
+// Shared tail of both mainloops, run by the 128 epilogue threads (tid 0..127): the partial tile
+// for EPI_PARTIAL; otherwise ticketing for split-K and argmax, then the epilogue. get(c0, v) fills
+// this thread's 16 accumulator values of columns c0..c0+15.
 template <typename T, int BN, int EPI, typename Get>
 JF_DEV void finish_tile(const GemmParams& p, Get get, float* xs, int* sflag, int n_tile, int split, int m_tile,
                         int tid) {
@@ -214,6 +218,22 @@ JF_DEV void finish_tile(const GemmParams& p, Get get, float* xs, int* sflag, int
   int ncols = p.M - m0;
   if (ncols > BN) ncols = BN;
   const int nchunks = (ncols + 15) >> 4;
+  if constexpr (EPI == EPI_PARTIAL) {
+    float* mine = p.ws + ((size_t)tile_lin * p.k_splits + split) * (size_t)BN * kTileN;
+    for (int c = 0; c < nchunks; ++c) {
+      float v[16];
+      get(c * 16, v);
+#pragma unroll
+      for (int j = 0; j < 16; ++j) mine[(c * 16 + j) * kTileN + tid] = v[j];
+    }
+  } else {
+    finish_tile_epi<T, BN, EPI>(p, get, xs, sflag, n_tile, split, m_tile, tid, n0, m0, tile_lin, nchunks);
+  }
+}
+
+template <typename T, int BN, int EPI, typename Get>
+JF_DEV void finish_tile_epi(const GemmParams& p, Get get, float* xs, int* sflag, int n_tile, int split, int m_tile,
+                            int tid, int n0, int m0, int tile_lin, int nchunks) {
   if (p.k_splits == 1) {
     for (int c = 0; c < nchunks; ++c) {
       float v[16];
@@ -550,6 +570,7 @@ cudaError_t launch_tc(const CUtensorMap& tmA, const CUtensorMap& tmB, const Gemm
     case EPI_QKV: return launch_tc_epi<BN, EPI_QKV>(tmA, tmB, p, st);
     case EPI_SWIGLU: return launch_tc_epi<BN, EPI_SWIGLU>(tmA, tmB, p, st);
     case EPI_ARGMAX: return launch_tc_epi<BN, EPI_ARGMAX>(tmA, tmB, p, st);
+    case EPI_PARTIAL: return launch_tc_epi<BN, EPI_PARTIAL>(tmA, tmB, p, st);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -562,7 +583,8 @@ cudaError_t prep_tc() {
   if ((e = cudaFuncSetAttribute(k_gemm_tc<BN, EPI_RESID>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm))) return e;
   if ((e = cudaFuncSetAttribute(k_gemm_tc<BN, EPI_QKV>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm))) return e;
   if ((e = cudaFuncSetAttribute(k_gemm_tc<BN, EPI_SWIGLU>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm))) return e;
-  return cudaFuncSetAttribute(k_gemm_tc<BN, EPI_ARGMAX>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+  if ((e = cudaFuncSetAttribute(k_gemm_tc<BN, EPI_ARGMAX>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm))) return e;
+  return cudaFuncSetAttribute(k_gemm_tc<BN, EPI_PARTIAL>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
 }
 
 }  // namespace

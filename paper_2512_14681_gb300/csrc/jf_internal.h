@@ -22,7 +22,10 @@ constexpr int kPage = 16;         // tokens per KV page
 constexpr int kTileN = 128;       // weight rows per GEMM tile (tcgen05 M)
 constexpr int kTileK = 64;        // K elements per GEMM pipeline stage
 constexpr int kAttnChunk = 128;   // keys per split-KV chunk, aligned to absolute positions
-constexpr int kAttnQRows = 64;    // (token, head) query rows per attention work unit
+constexpr int kAttnQRows = 128;   // (token, head) query rows per attention work unit
+constexpr int kAttnLanes = 8;     // chunk lanes per unit (c mod 8); one CTA of an 8-CTA cluster each
+constexpr int kAttnLaneChunks = 128;  // chunks per lane the kernel can stage page ids for
+constexpr int kAttnMaxCtx = kAttnChunk * kAttnLanes * kAttnLaneChunks;  // 131072 key positions
 constexpr int kMaxSeqs = 64;
 constexpr int kMaxChains = 256;
 
@@ -33,15 +36,22 @@ struct Chain {
   int seq, row0, nrows, pos0;
 };
 
-// Attention work decomposition computed on the device once per forward.
+// Attention work unit: (chain, KV head, tile of 64 (token, head) query rows), its chain resolved;
+// `pad` is nonzero for a unit that exists.
 struct AttnUnit {
-  int chain, kvh, qt, n_chunks, slot0;
-};
-struct AttnPlan {
-  int n_units, n_items, n_slots, pad;
+  int seq, row0, nrows, pos0, kvh, qt, n_chunks, pad;
 };
 
-enum EpiKind : int { EPI_STORE = 0, EPI_RESID = 1, EPI_QKV = 2, EPI_SWIGLU = 3, EPI_ARGMAX = 4 };
+// EPI_PARTIAL: the tile's (split's) fp32 partial sums go to the workspace and the consumer kernel
+// adds the k_splits partials of an element in split order (no ticket, no last-CTA reduction).
+enum EpiKind : int { EPI_STORE = 0, EPI_RESID = 1, EPI_QKV = 2, EPI_SWIGLU = 3, EPI_ARGMAX = 4, EPI_PARTIAL = 5 };
+
+// Where the consumer of an EPI_PARTIAL projection finds element (m, n): partial s lives at
+// ws[((n / 128 * m_tiles + m / bn) * k_splits + s) * bn * 128 + (m % bn) * 128 + n % 128].
+struct SplitPartials {
+  const float* ws;
+  int k_splits, m_tiles, bn;
+};
 
 struct GemmEpi {
   int kind;
@@ -93,12 +103,6 @@ struct AttnParams {
   const int* seq_len;   // committed length per sequence
   const Chain* chains;
   const int* n_chains_dev;
-  const AttnPlan* plan;
-  const AttnUnit* units;
-  const int2* items;    // (unit, chunk)
-  float* ws_o;          // [slot][64][hd]
-  float* ws_ml;         // [slot][64][2]
-  int* unit_counter;    // [max_units]
   void* out;            // [R][Hq*hd]
   int Hq, Hkv, hd;
   float scale_log2;     // log2(e) / sqrt(hd)

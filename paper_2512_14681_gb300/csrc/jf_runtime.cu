@@ -22,14 +22,12 @@ cudaError_t launch_fill_f32(float* p, long long n, float v, cudaStream_t st);
 cudaError_t launch_rope_table(float2* tab, int n_pos, int half, double theta, cudaStream_t st);
 cudaError_t launch_embed(const void* E, bool is_bf16, const int* tok, float* x, int rows, int d, int V, int* err,
                          cudaStream_t st);
-cudaError_t launch_rmsnorm(const float* x, const float* gain, void* y, bool is_bf16, int rows, int d, float eps,
-                           cudaStream_t st);
-cudaError_t launch_attn_plan(const Chain* chains, const int* n_chains_dev, int Hq, int Hkv, AttnPlan* plan,
-                             AttnUnit* units, int2* items, int max_units, int max_items, int max_slots, int* err,
-                             cudaStream_t st);
-cudaError_t launch_attn_bf16(const AttnParams& a, int grid, cudaStream_t st);
+cudaError_t launch_rmsnorm(float* x, const float* gain, void* y, bool is_bf16, int rows, int d, float eps,
+                           const SplitPartials* acc, int row0, cudaStream_t st);
+cudaError_t launch_qkv_finish(const SplitPartials& sp, const int* pos, const float2* rope, void* q, void* k, void* v,
+                              int M, int Hq, int Hkv, cudaStream_t st);
+cudaError_t launch_attn_bf16(const AttnParams& a, int units_bound, cudaStream_t st);
 cudaError_t launch_attn_f32(const AttnParams& a, int n_rows, cudaStream_t st);
-cudaError_t launch_attn_combine(const AttnParams& a, int max_units, cudaStream_t st);
 size_t attn_bf16_smem_bytes();
 cudaError_t gemm_prepare();
 cudaError_t attn_prepare();
@@ -92,7 +90,7 @@ struct Dims {
   int es;
   bool bf16;
   int R, S, max_ctx, pps, n_pages, logits_rows;
-  int max_chains, max_units, max_items, max_slots;
+  int max_chains, max_units;
   int n_vtiles;
 };
 
@@ -112,7 +110,6 @@ struct Offsets {
   size_t k_pages, v_pages, page_table, seq_len, commit;
   size_t k_inf, v_inf, x, h, q, att, act;
   size_t tok, pos, gpred, top2, chains, n_chains;
-  size_t plan, units, items, unit_counter, ws_o, ws_ml;
   size_t gemm_ws, gemm_counter, am_v1, am_i1, am_v2, am_counter;
   size_t logits, err;
   size_t gen_state, gen_out, gen_truth, gen_log, gen_q0, gen_plast, res, step_blocks, step_res, committed;
@@ -142,6 +139,10 @@ jf_status make_dims(const jf_model_config* m, const jf_runtime_config* rt, Dims*
     *why = "runtime capacity out of range (max_seqs 1..64, max_ctx >= 16, max_rows 1..4096, logits_rows <= max_rows)";
     return JF_EINVAL;
   }
+  if (m->dtype == JF_BF16 && rt->max_ctx > kAttnMaxCtx - kAttnChunk) {
+    *why = "max_ctx above the bf16 attention's page-id staging capacity (130944 positions)";
+    return JF_EINVAL;
+  }
   D->L = m->n_layers; D->d = m->d_model; D->Hq = m->n_heads; D->Hkv = m->n_kv_heads; D->hd = m->head_dim;
   D->F = m->d_ff; D->V = m->vocab;
   D->nq = D->Hq * D->hd; D->nkv = D->Hkv * D->hd; D->nqkv = D->nq + 2 * D->nkv; D->G = D->Hq / D->Hkv;
@@ -151,11 +152,8 @@ jf_status make_dims(const jf_model_config* m, const jf_runtime_config* rt, Dims*
   D->max_chains = std::min(kMaxChains, D->S * 5 + 1);
   if (D->bf16) {
     D->max_units = D->Hkv * (cdiv((long long)D->R * D->G, kAttnQRows) + D->max_chains);
-    const int chunks = cdiv(D->max_ctx, kAttnChunk) + 1;
-    D->max_items = D->max_units * chunks;
-    D->max_slots = D->max_items;
   } else {
-    D->max_units = D->max_items = D->max_slots = 1;
+    D->max_units = 1;
   }
   D->n_vtiles = cdiv(D->V, kTileN);
   return JF_OK;
@@ -169,7 +167,8 @@ size_t gemm_ws_floats(const Dims& D) {
   for (int i = 0; i < 5; ++i) {
     const int nt = cdiv(N[i], kTileN), kb = cdiv(K[i], kTileK);
     const int sp = splits_for(nt, kb);
-    if (sp <= 1) continue;
+    // QKV, O and down always leave partial tiles for their consumer; the others only when split
+    if (sp <= 1 && (i == 2 || i == 4)) continue;
     mx = std::max(mx, (size_t)sp * nt * ((size_t)D.R + 256) * kTileN);
   }
   return mx;
@@ -211,12 +210,6 @@ Offsets plan_offsets(const Dims& D) {
   o.top2 = p.take((size_t)D.R * 8);
   o.chains = p.take((size_t)kMaxChains * sizeof(Chain));
   o.n_chains = p.take(16);
-  o.plan = p.take(sizeof(AttnPlan));
-  o.units = p.take((size_t)D.max_units * sizeof(AttnUnit));
-  o.items = p.take((size_t)D.max_items * sizeof(int2));
-  o.unit_counter = p.take((size_t)D.max_units * 4);
-  o.ws_o = p.take(D.bf16 ? (size_t)D.max_slots * kAttnQRows * D.hd * 4 : 16, 1024);
-  o.ws_ml = p.take(D.bf16 ? (size_t)D.max_slots * kAttnQRows * 2 * 4 : 16);
   o.gemm_ws_bytes = gemm_ws_floats(D) * 4;
   o.gemm_ws = p.take(std::max<size_t>(o.gemm_ws_bytes, 16), 1024);
   const int max_mt = cdiv(D.R, 16) + 1;
@@ -290,11 +283,7 @@ struct jf_ctx {
   float* top2;
   Chain* chains;
   int* n_chains;
-  AttnPlan* plan;
-  AttnUnit* units;
-  int2* items;
-  int* unit_counter;
-  float *ws_o, *ws_ml;
+  int chains_bound = 1;  // most chains the next forward can have (sizes the attention launch)
   float* gemm_ws;
   int* gemm_counter;
   float *am_v1, *am_v2;
@@ -479,48 +468,51 @@ cudaError_t enqueue_forward(jf_ctx* c, int M, LmMode lm) {
   e = launch_embed(c->w_embed, D.bf16, c->tok, c->x, M, D.d, D.V, c->err, c->st);
   prof_end(c);
   if (e != cudaSuccess) return e;
-  if (D.bf16) {
-    prof_begin(c, PC_OTHER);
-    e = launch_attn_plan(c->chains, c->n_chains, D.Hq, D.Hkv, c->plan, c->units, c->items, D.max_units, D.max_items,
-                         D.max_slots, c->err, c->st);
-    prof_end(c);
-    if (e != cudaSuccess) return e;
-  }
   const size_t inf_layer = (size_t)D.R * D.nkv * D.es;
   const size_t kv_layer = (size_t)D.n_pages * D.Hkv * kPage * D.hd * D.es;
+  // bf16: the QKV, O and down projections leave split-K partial tiles; the QKV finish kernel and
+  // the following RMSNorms add them (split order) instead of a last-CTA reduction in the GEMM
+  const bool partials = D.bf16;
+  const bool qkv_partial = partials && D.hd == kTileN;
+  auto split_parts = [&](int N, int K) {
+    const int bn = gemm_bn_for(M);
+    return SplitPartials{c->gemm_ws, splits_for(cdiv(N, kTileN), cdiv(K, kTileK)), cdiv(M, bn), bn};
+  };
+  const SplitPartials sp_qkv = split_parts(D.nqkv, D.d), sp_o = split_parts(D.d, D.nq), sp_dn = split_parts(D.d, D.F);
   for (int l = 0; l < D.L; ++l) {
     LayerW& w = c->layers[l];
     char* kinf = reinterpret_cast<char*>(c->k_inf) + l * inf_layer;
     char* vinf = reinterpret_cast<char*>(c->v_inf) + l * inf_layer;
     prof_begin(c, PC_NORM);
-    e = launch_rmsnorm(c->x, w.g_attn, c->h, D.bf16, M, D.d, eps, c->st);
+    e = launch_rmsnorm(c->x, w.g_attn, c->h, D.bf16, M, D.d, eps, (partials && l > 0) ? &sp_dn : nullptr, 0, c->st);
     prof_end(c);
     if (e != cudaSuccess) return e;
     GemmEpi ep = {};
-    ep.kind = EPI_QKV;
+    ep.kind = qkv_partial ? EPI_PARTIAL : EPI_QKV;
     ep.q_out = c->q; ep.k_out = kinf; ep.v_out = vinf;
     ep.n_q = D.nq; ep.n_kv = D.nkv; ep.head_dim = D.hd;
     ep.pos = c->pos; ep.rope = c->rope;
     if ((e = gemm(c, w.tm_qkv, w.qkv, c->h, D.nqkv, D.d, M, ep, PC_QKV)) != cudaSuccess) return e;
+    if (qkv_partial) {
+      prof_begin(c, PC_QKV);
+      e = launch_qkv_finish(sp_qkv, c->pos, c->rope, c->q, kinf, vinf, M, D.Hq, D.Hkv, c->st);
+      prof_end(c);
+      if (e != cudaSuccess) return e;
+    }
     AttnParams a = {};
     a.q = c->q; a.k_inf = kinf; a.v_inf = vinf;
     a.k_pages = reinterpret_cast<char*>(c->k_pages) + l * kv_layer;
     a.v_pages = reinterpret_cast<char*>(c->v_pages) + l * kv_layer;
     a.page_table = c->page_table; a.pages_per_seq = D.pps; a.n_pages = D.n_pages;
     a.seq_len = c->seq_len; a.chains = c->chains; a.n_chains_dev = c->n_chains;
-    a.plan = c->plan; a.units = c->units; a.items = c->items;
-    a.ws_o = c->ws_o; a.ws_ml = c->ws_ml; a.unit_counter = c->unit_counter;
     a.out = c->att; a.Hq = D.Hq; a.Hkv = D.Hkv; a.hd = D.hd;
     a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)D.hd));
     a.err = c->err;
     prof_begin(c, PC_ATTN);
     if (D.bf16) {
-      e = launch_attn_bf16(a, 2 * c->num_sms, c->st);
-      prof_end(c);
       // units of this forward are bounded by its rows: every chain adds at most one partial tile
-      const int units_bound = std::min(D.max_units, D.Hkv * (cdiv((long long)M * D.G, kAttnQRows) + D.max_chains));
-      prof_begin(c, PC_COMBINE);
-      if (e == cudaSuccess) e = launch_attn_combine(a, units_bound, c->st);
+      const int units_bound = std::min(D.max_units, D.Hkv * (cdiv((long long)M * D.G, kAttnQRows) + c->chains_bound));
+      e = launch_attn_bf16(a, units_bound, c->st);
       prof_end(c);
     } else {
       e = launch_attn_f32(a, M, c->st);
@@ -528,10 +520,10 @@ cudaError_t enqueue_forward(jf_ctx* c, int M, LmMode lm) {
     }
     if (e != cudaSuccess) return e;
     GemmEpi er = {};
-    er.kind = EPI_RESID; er.x = c->x; er.ldx = D.d;
+    er.kind = partials ? EPI_PARTIAL : EPI_RESID; er.x = c->x; er.ldx = D.d;
     if ((e = gemm(c, w.tm_o, w.o, c->att, D.d, D.nq, M, er, PC_OPROJ)) != cudaSuccess) return e;
     prof_begin(c, PC_NORM);
-    e = launch_rmsnorm(c->x, w.g_mlp, c->h, D.bf16, M, D.d, eps, c->st);
+    e = launch_rmsnorm(c->x, w.g_mlp, c->h, D.bf16, M, D.d, eps, partials ? &sp_o : nullptr, 0, c->st);
     prof_end(c);
     if (e != cudaSuccess) return e;
     GemmEpi es = {};
@@ -540,13 +532,13 @@ cudaError_t enqueue_forward(jf_ctx* c, int M, LmMode lm) {
     if ((e = gemm(c, w.tm_dn, w.dn, c->act, D.d, D.F, M, er, PC_DOWN)) != cudaSuccess) return e;
   }
   if (lm == LM_NONE) {
-    c->launches += 1 + (D.bf16 ? 1 : 0) + (D.bf16 ? 8LL : 7LL) * D.L;
+    c->launches += 1 + (qkv_partial ? 8LL : 7LL) * D.L;
     return cudaSuccess;
   }
   const int lm_rows = (lm == LM_LAST) ? 1 : M;
-  const float* x_lm = c->x + (size_t)(M - lm_rows) * D.d;
   prof_begin(c, PC_NORM);
-  e = launch_rmsnorm(x_lm, c->g_final, c->h, D.bf16, lm_rows, D.d, eps, c->st);
+  e = launch_rmsnorm(c->x, c->g_final, c->h, D.bf16, lm_rows, D.d, eps, (partials && D.L > 0) ? &sp_dn : nullptr,
+                     M - lm_rows, c->st);
   prof_end(c);
   if (e != cudaSuccess) return e;
   GemmEpi el = {};
@@ -557,7 +549,7 @@ cudaError_t enqueue_forward(jf_ctx* c, int M, LmMode lm) {
   } else {
     el.kind = EPI_STORE; el.y = c->logits; el.ldy = D.V;
   }
-  c->launches += 1 + (D.bf16 ? 1 : 0) + (D.bf16 ? 8LL : 7LL) * D.L + 2;
+  c->launches += 1 + (qkv_partial ? 8LL : 7LL) * D.L + 2;
   return gemm(c, c->tm_lm, c->w_lm, c->h, D.V, D.d, lm_rows, el, PC_LMHEAD);
 }
 
@@ -573,6 +565,7 @@ jf_status upload_chain(jf_ctx* c, int seq, int P, int M, const int32_t* tokens_h
   CK(cudaMemcpyAsync(c->chains, &ch, sizeof(Chain), cudaMemcpyHostToDevice, c->st));
   CK(cudaMemcpyAsync(c->n_chains, &one, 4, cudaMemcpyHostToDevice, c->st));
   CK(cudaStreamSynchronize(c->st));
+  c->chains_bound = 1;
   return JF_OK;
 }
 
@@ -800,6 +793,7 @@ jf_status generate_impl(jf_ctx* c, int n_seqs, const int32_t* const* h_prompts, 
   g.truth_len = p.init == JF_INIT_INJECT ? p.truth_len : 0;
   g.state_stride = L.total;
   g.max_rows = D.R; g.max_chains = D.max_chains; g.max_ctx = D.max_ctx;
+  c->chains_bound = std::min(D.max_chains, n_seqs * (1 + g.C));
   g.out_tokens = c->gen_out; g.iter_log = c->gen_log; g.max_iters = D.max_ctx;
   CK(launch_gen_init(g, c->gen_state, c->gen_q0, c->seq_len, c->gen_plast, c->tok, c->pos, c->chains, c->n_chains,
                      c->res_dev, c->err, c->st));
@@ -933,12 +927,6 @@ jf_status jf_create(const jf_model_config* model, const jf_runtime_config* rt, j
   c->top2 = at<float>(c, O.top2);
   c->chains = at<Chain>(c, O.chains);
   c->n_chains = at<int>(c, O.n_chains);
-  c->plan = at<AttnPlan>(c, O.plan);
-  c->units = at<AttnUnit>(c, O.units);
-  c->items = at<int2>(c, O.items);
-  c->unit_counter = at<int>(c, O.unit_counter);
-  c->ws_o = at<float>(c, O.ws_o);
-  c->ws_ml = at<float>(c, O.ws_ml);
   c->gemm_ws = at<float>(c, O.gemm_ws);
   c->gemm_counter = at<int>(c, O.gemm_counter);
   c->am_v1 = at<float>(c, O.am_v1);
@@ -966,7 +954,6 @@ jf_status jf_create(const jf_model_config* model, const jf_runtime_config* rt, j
   };
   zero(O.seq_len, (size_t)D.S * 4);
   zero(O.commit, (size_t)D.S * sizeof(CommitInfo));
-  zero(O.unit_counter, (size_t)D.max_units * 4);
   zero(O.gemm_counter, (O.am_v1 - O.gemm_counter));
   zero(O.am_counter, (size_t)(cdiv(D.R, 16) + 1) * 4);
   zero(O.err, 16);
@@ -1274,6 +1261,7 @@ jf_status jf_jacobi_step(jf_ctx* c, int seq, int n_blocks, const jf_block* block
   CK(cudaMemcpyAsync(c->n_chains, &nch, 4, cudaMemcpyHostToDevice, c->st));
   CK(cudaMemcpyAsync(c->sb_dev, &sb, sizeof(sb), cudaMemcpyHostToDevice, c->st));
   CK(cudaStreamSynchronize(c->st));
+  c->chains_bound = nch;
   CK(enqueue_forward(c, total, LM_ARGMAX));
   CK(launch_step_accept(c->sb_dev, c->tok, c->gpred, c->committed_dev, c->commit, c->sres_dev, c->err, c->st));
   CK(launch_commit(c->commit + seq, 1, D.L, c->k_inf, c->v_inf, c->k_pages, c->v_pages,

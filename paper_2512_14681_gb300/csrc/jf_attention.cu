@@ -14,9 +14,10 @@
 // chunk c belongs to lane c mod 8. A unit runs on one 8-CTA cluster: CTA j walks the chunks of
 // lane j in increasing order, 64 keys at a time, with one online-softmax state per row (QK^T and
 // PV on mma.sync.m16n8k16, keys staged by cp.async into XOR-swizzled shared memory, the next chunk
-// in flight while the current one computes). Each warp then stores its 16 rows' lane state into
-// the shared memory of the CTA that owns those rows, and after one cluster barrier each CTA folds
-// its rows' 8 lane states in lane order. The tree depends only on absolute key positions, never on
+// in flight while the current one computes). Each warp then stages its 16 rows' lane state as one
+// block and sends it with a bulk copy into the shared memory of the CTA that owns those rows;
+// once its 8 blocks have arrived (mbarrier transaction count) each CTA folds its rows' 8 lane
+// states in lane order. The tree depends only on absolute key positions, never on
 // how many rows share the forward or how many chunks a unit has, so a row's result is the same in
 // every batch.
 // fp32 path: one warp per (row, head), keys in absolute order, online softmax in fp32.
@@ -34,9 +35,13 @@ constexpr int TILE_BYTES = SUB * ROW_BYTES;  // 16 KB
 constexpr int STAGE_BYTES = 2 * NSUB * TILE_BYTES;     // K and V of one chunk: 64 KB
 constexpr int ROWS_PER_CTA = kAttnQRows / kAttnLanes;  // rows each CTA of a cluster folds (16)
 constexpr int Q_BYTES = kAttnQRows * ROW_BYTES;         // staged queries: 32 KB
-constexpr int RECV_BYTES = ROWS_PER_CTA * kAttnLanes * HD * 4;  // received lane states: 64 KB
+// lane-state block of 16 rows: O [16][128], then m [16], then l [16] (fp32)
+constexpr int BLOCK_FLOATS = ROWS_PER_CTA * HD + 2 * ROWS_PER_CTA;
+constexpr int BLOCK_BYTES = BLOCK_FLOATS * 4;          // 8320 B
+constexpr int RECV_BYTES = kAttnLanes * BLOCK_BYTES;   // the 8 lanes' blocks of this CTA's rows
 constexpr int REGION0 = RECV_BYTES > Q_BYTES ? RECV_BYTES : Q_BYTES;  // queries, later the lane states
-constexpr int ATT_SMEM = REGION0 + 2 * STAGE_BYTES;   // 192 KB
+constexpr int ATT_SMEM = REGION0 + 2 * STAGE_BYTES;   // 193 KB
+static_assert(BLOCK_BYTES % 16 == 0 && kAttnLanes * BLOCK_BYTES <= 2 * STAGE_BYTES, "lane-state blocks");
 
 JF_DEV uint32_t swz(int r, int c16) { return (uint32_t)(r * ROW_BYTES + ((c16 ^ (r & 7)) << 4)); }
 
@@ -126,9 +131,9 @@ constexpr int ATT_THREADS = 256;
 __global__ void __launch_bounds__(ATT_THREADS, 1) k_attn_bf16(const AttnParams a) {
   extern __shared__ __align__(128) uint8_t sm[];
   uint8_t* sQ = sm;                                  // 128 x 256 B, free once the queries are in registers
-  float* recv = reinterpret_cast<float*>(sm);        // [16 rows][8 lanes][128], aliases sQ
-  uint8_t* stage0 = sm + REGION0;                    // chunk stages, 64 KB each
-  __shared__ float recv_m[ROWS_PER_CTA * kAttnLanes], recv_l[ROWS_PER_CTA * kAttnLanes];
+  float* recv = reinterpret_cast<float*>(sm);        // [8 lanes][block], aliases sQ
+  uint8_t* stage0 = sm + REGION0;                    // chunk stages, 64 KB each; outgoing blocks at the end
+  __shared__ __align__(8) uint64_t recv_bar;
   __shared__ int s_rowpos[kAttnQRows];
   __shared__ int s_page[kAttnLaneChunks * (kAttnChunk / kPage)];
   __shared__ AttnUnit s_unit;
@@ -138,6 +143,11 @@ __global__ void __launch_bounds__(ATT_THREADS, 1) k_attn_bf16(const AttnParams a
   const int ui = (int)cluster_id_x();
   const int G = a.Hq / a.Hkv;
   pdl_launch_dependents();  // the next kernel may launch now
+  if (tid == 0) {
+    // receives the 8 lane-state blocks of this CTA's rows (one bulk copy from each CTA)
+    mbar_init(smem_u32(&recv_bar), 1);
+    fence_mbar_init();
+  }
   // Before the dependency wait: the chain table, the page table and the cached keys were written
   // by host copies or by an earlier graph launch, all complete before this forward began.
   // Unit ui of the forward: chains in order, then KV heads, then 128-row query tiles.
@@ -238,7 +248,7 @@ __global__ void __launch_bounds__(ATT_THREADS, 1) k_attn_bf16(const AttnParams a
         const int r = warp * 16 + (lane & 15), c = kk * 2 + (lane >> 4);
         ldsm_x4(smem_u32(sQ) + swz(r, c), qf[kk][0], qf[kk][1], qf[kk][2], qf[kk][3]);
       }
-      cluster_arrive_relaxed();  // this CTA's query staging is no longer read
+      cluster_arrive();  // this CTA's query staging is no longer read; its receive barrier is initialised
     }
     const int chunk = sub_of(t);
     uint8_t* stage = stage0 + (t & 1) * STAGE_BYTES;
@@ -328,41 +338,50 @@ __global__ void __launch_bounds__(ATT_THREADS, 1) k_attn_bf16(const AttnParams a
       cp_async_commit();
     }
   }
-  if (n_steps == 0) cluster_arrive_relaxed();
+  if (n_steps == 0) cluster_arrive();
 #pragma unroll
   for (int sh = 1; sh <= 2; sh <<= 1) {
     l_lo += __shfl_xor_sync(0xffffffffu, l_lo, sh);
     l_hi += __shfl_xor_sync(0xffffffffu, l_hi, sh);
   }
-  // this warp's lane state goes to CTA `warp`, owner of rows 16w .. 16w+15 (r_lo: row lane/4, r_hi: +8)
-  cluster_wait();  // every CTA of the cluster has its queries in registers: the receive buffers are free
+  // this warp's lane state (rows 16w .. 16w+15) is staged as one block and copied into CTA w
   {
+    float* blk = reinterpret_cast<float*>(stage0) + warp * BLOCK_FLOATS;  // stages are free after the loop
     const int d0 = 2 * (lane & 3);
     const int lr = lane >> 2;
-    const uint32_t peer = (uint32_t)warp;
-    const uint32_t o_lo = dsmem_addr(smem_u32(recv + (lr * kAttnLanes + j) * HD + d0), peer);
-    const uint32_t o_hi = dsmem_addr(smem_u32(recv + ((lr + 8) * kAttnLanes + j) * HD + d0), peer);
 #pragma unroll
     for (int i = 0; i < HD / 8; ++i) {
-      dsmem_st_f32x2(o_lo + i * 32, o[i][0], o[i][1]);
-      dsmem_st_f32x2(o_hi + i * 32, o[i][2], o[i][3]);
+      *reinterpret_cast<float2*>(blk + lr * HD + i * 8 + d0) = make_float2(o[i][0], o[i][1]);
+      *reinterpret_cast<float2*>(blk + (lr + 8) * HD + i * 8 + d0) = make_float2(o[i][2], o[i][3]);
     }
     if ((lane & 3) == 0) {
-      dsmem_st_f32(dsmem_addr(smem_u32(recv_m + lr * kAttnLanes + j), peer), m_lo);
-      dsmem_st_f32(dsmem_addr(smem_u32(recv_l + lr * kAttnLanes + j), peer), l_lo);
-      dsmem_st_f32(dsmem_addr(smem_u32(recv_m + (lr + 8) * kAttnLanes + j), peer), m_hi);
-      dsmem_st_f32(dsmem_addr(smem_u32(recv_l + (lr + 8) * kAttnLanes + j), peer), l_hi);
+      blk[ROWS_PER_CTA * HD + lr] = m_lo;
+      blk[ROWS_PER_CTA * HD + lr + 8] = m_hi;
+      blk[ROWS_PER_CTA * HD + ROWS_PER_CTA + lr] = l_lo;
+      blk[ROWS_PER_CTA * HD + ROWS_PER_CTA + lr + 8] = l_hi;
+    }
+    fence_proxy_async_smem();  // make the block visible to the bulk-copy engine
+    __syncwarp();
+    if (tid == 0) mbar_arrive_expect_tx(smem_u32(&recv_bar), (uint32_t)RECV_BYTES);
+    cluster_wait();  // every CTA of the cluster has its queries in registers: the receive buffers are free
+    if (lane == 0) {
+      const uint32_t peer = (uint32_t)warp;
+      bulk_copy_to_cluster(dsmem_addr(smem_u32(recv + j * BLOCK_FLOATS), peer), smem_u32(blk), (uint32_t)BLOCK_BYTES,
+                           dsmem_addr(smem_u32(&recv_bar), peer));
     }
   }
-  // every lane state of this CTA's rows has arrived; no shared memory is accessed remotely after this
-  cluster_sync();
+  // all 8 blocks of this CTA's rows have arrived
+  const bool got = mbar_wait_cluster_bounded(smem_u32(&recv_bar), 0u, JF_WAIT_LIMIT_NS);
+  if (!got && tid == 0) jf_set_error(a.err, JF_DERR_TIMEOUT_TMA);
   // fold of rows 16j .. 16j+15 over the 8 lanes in order; thread = (row, 8 of the 128 dims)
   {
     const int lr = tid >> 4, r = j * ROWS_PER_CTA + lr;
     const int d = (tid & 15) * 8;
-    if (r < qrows) {
-      const float* ro = recv + lr * kAttnLanes * HD + d;
-      float M = recv_m[lr * kAttnLanes], L = recv_l[lr * kAttnLanes];
+    if (got && r < qrows) {
+      const float* ro = recv + lr * HD + d;
+      const float* rm = recv + ROWS_PER_CTA * HD + lr;
+      const float* rl = rm + ROWS_PER_CTA;
+      float M = rm[0], L = rl[0];
       float acc[8];
       {
         const float4 x0 = *reinterpret_cast<const float4*>(ro), x1 = *reinterpret_cast<const float4*>(ro + 4);
@@ -372,11 +391,11 @@ __global__ void __launch_bounds__(ATT_THREADS, 1) k_attn_bf16(const AttnParams a
 #pragma unroll
       for (int q = 1; q < kAttnLanes; ++q) {
         float wa, wb, mm;
-        fold_weights(M, recv_m[lr * kAttnLanes + q], wa, wb, mm);
-        const float4 x0 = *reinterpret_cast<const float4*>(ro + q * HD);
-        const float4 x1 = *reinterpret_cast<const float4*>(ro + q * HD + 4);
+        fold_weights(M, rm[q * BLOCK_FLOATS], wa, wb, mm);
+        const float4 x0 = *reinterpret_cast<const float4*>(ro + q * BLOCK_FLOATS);
+        const float4 x1 = *reinterpret_cast<const float4*>(ro + q * BLOCK_FLOATS + 4);
         M = mm;
-        L = wa * L + wb * recv_l[lr * kAttnLanes + q];
+        L = wa * L + wb * rl[q * BLOCK_FLOATS];
         acc[0] = wa * acc[0] + wb * x0.x; acc[1] = wa * acc[1] + wb * x0.y;
         acc[2] = wa * acc[2] + wb * x0.z; acc[3] = wa * acc[3] + wb * x0.w;
         acc[4] = wa * acc[4] + wb * x1.x; acc[5] = wa * acc[5] + wb * x1.y;
@@ -389,6 +408,8 @@ __global__ void __launch_bounds__(ATT_THREADS, 1) k_attn_bf16(const AttnParams a
                                                   pack_bf16(acc[4] * il, acc[5] * il), pack_bf16(acc[6] * il, acc[7] * il));
     }
   }
+  // every copy out of this CTA's shared memory has landed (each CTA has received all it was sent)
+  cluster_sync();
 }
 
 // fp32 path: one warp per (row, query head); keys in absolute order, 32 at a time.

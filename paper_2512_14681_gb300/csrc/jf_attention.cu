@@ -128,7 +128,9 @@ constexpr int ATT_THREADS = 256;
 // 8 warps: warp w owns query rows 16w .. 16w+15 of the tile and walks the lane's chunks, 64 keys
 // at a time, with one online-softmax state; at the end it stores that lane state of its 16 rows
 // into CTA w of the cluster, which folds rows 16w .. 16w+15 over the 8 lanes.
-__global__ void __launch_bounds__(ATT_THREADS, 1) k_attn_bf16(const AttnParams a) {
+// At most 200 registers a thread (51,200 of the SM's 65,536): the CTAs of the QKV finish kernel
+// still resident on an SM leave room for this one, so the clusters are placed while it runs.
+__global__ void __maxnreg__(200) k_attn_bf16(const AttnParams a) {
   extern __shared__ __align__(128) uint8_t sm[];
   uint8_t* sQ = sm;                                  // 128 x 256 B, free once the queries are in registers
   float* recv = reinterpret_cast<float*>(sm);        // [8 lanes][block], aliases sQ

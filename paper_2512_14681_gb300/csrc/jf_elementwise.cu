@@ -80,13 +80,28 @@ __global__ void k_embed(const T* __restrict__ E, const int* __restrict__ tok, fl
 }
 
 // y[r, :] = x[r, :] / sqrt(mean(x[r, :]^2) + eps) * gain, rounded to the activation type.
-// One CTA per row; the row stays in registers (float4, up to 8 per thread: d <= 8192), so x is
-// read once. The reduction order is fixed by d alone.
+// One CTA of 512 threads per row; the row stays in registers (float4, up to 4 per thread:
+// d <= 8192), so x is read once. The reduction order is fixed by d alone.
 // ACC: the residual update of the preceding projection is finished here first: the k_splits
 // partial sums of x's increment (EPI_PARTIAL) are added in split order, x += that sum is written
-// back, and the norm is taken of the updated row. Rows are row0 + blockIdx.x.
-constexpr int NORM_THREADS = 256;
-constexpr int NORM_VEC = 8;
+// back, and the norm is taken of the updated row. Every load of a row is issued before the first
+// add (the row's bytes are one round trip), which is what bounds this kernel. Rows are
+// row0 + blockIdx.x.
+constexpr int NORM_THREADS = 512;
+constexpr int NORM_VEC = 4;
+constexpr int kMaxPartialSplits = 8;  // the host never splits K more than this
+
+// L2-cached 16-byte load that yields zeros when `pred` is false. Volatile: a run of these is
+// issued back to back, so all of them are in flight before the first use.
+__device__ __forceinline__ float4 ldcg4_if(const float* p, bool pred) {
+  float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+  asm volatile(
+      "{\n\t.reg .pred q;\n\tsetp.ne.b32 q, %5, 0;\n\t@q ld.global.cg.v4.f32 {%0,%1,%2,%3}, [%4];\n\t}"
+      : "+f"(v.x), "+f"(v.y), "+f"(v.z), "+f"(v.w)
+      : "l"(p), "r"((int)pred)
+      : "memory");
+  return v;
+}
 
 __device__ __forceinline__ void store4(float* y, float4 v) { *reinterpret_cast<float4*>(y) = v; }
 __device__ __forceinline__ void store4(bf16* y, float4 v) {
@@ -108,28 +123,51 @@ __global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(float* __restrict__ x,
   const int nv = d >> 2;
   float4* xr = reinterpret_cast<float4*>(x + (size_t)r * d);
   float4 v[NORM_VEC];
-  float ss = 0.f;
 #pragma unroll
   for (int j = 0; j < NORM_VEC; ++j) {
     const int i = threadIdx.x + j * NORM_THREADS;
     v[j] = (i < nv) ? xr[i] : make_float4(0.f, 0.f, 0.f, 0.f);
-    if constexpr (ACC) {
-      if (i < nv) {
+  }
+  if constexpr (ACC) {
+    // two vectors' partials (and the row itself, above) in flight together
+#pragma unroll
+    for (int j0 = 0; j0 < NORM_VEC; j0 += 2) {
+      if (j0 * NORM_THREADS >= nv) break;
+      float4 q[2][kMaxPartialSplits];
+#pragma unroll
+      for (int jj = 0; jj < 2; ++jj) {
+        const int i = threadIdx.x + (j0 + jj) * NORM_THREADS;
         const int n = 4 * i;
         const float* base = sp.ws + ((size_t)((n >> 7) * sp.m_tiles + r / sp.bn) * sp.k_splits * sp.bn +
                                      (size_t)(r % sp.bn)) * 128 + (n & 127);
+#pragma unroll
+        for (int s = 0; s < kMaxPartialSplits; ++s)
+          q[jj][s] = ldcg4_if(base + (size_t)s * sp.bn * 128, i < nv && s < sp.k_splits);
+      }
+#pragma unroll
+      for (int jj = 0; jj < 2; ++jj) {
+        const int i = threadIdx.x + (j0 + jj) * NORM_THREADS;
         float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int s = 0; s < sp.k_splits; ++s) {
-          const float4 q = __ldcg(reinterpret_cast<const float4*>(base + (size_t)s * sp.bn * 128));
-          acc.x += q.x;
-          acc.y += q.y;
-          acc.z += q.z;
-          acc.w += q.w;
+#pragma unroll
+        for (int s = 0; s < kMaxPartialSplits; ++s) {
+          if (s < sp.k_splits) {
+            acc.x += q[jj][s].x;
+            acc.y += q[jj][s].y;
+            acc.z += q[jj][s].z;
+            acc.w += q[jj][s].w;
+          }
         }
-        v[j] = make_float4(v[j].x + acc.x, v[j].y + acc.y, v[j].z + acc.z, v[j].w + acc.w);
-        xr[i] = v[j];
+        const int j = j0 + jj;
+        if (i < nv) {
+          v[j] = make_float4(v[j].x + acc.x, v[j].y + acc.y, v[j].z + acc.z, v[j].w + acc.w);
+          xr[i] = v[j];
+        }
       }
     }
+  }
+  float ss = 0.f;
+#pragma unroll
+  for (int j = 0; j < NORM_VEC; ++j) {
     ss = fmaf(v[j].x, v[j].x, ss);
     ss = fmaf(v[j].y, v[j].y, ss);
     ss = fmaf(v[j].z, v[j].z, ss);
@@ -173,13 +211,20 @@ __global__ void __launch_bounds__(128) k_qkv_finish(SplitPartials sp, const int*
   const int m = job / slots, hs = job % slots;
   const float* base = sp.ws + ((size_t)(hs * sp.m_tiles + m / sp.bn) * sp.k_splits * sp.bn + (size_t)(m % sp.bn)) * 128 +
                       lane * 4;
+  // all partials in flight at once, then added in split order
+  float4 t[kMaxPartialSplits];
+#pragma unroll
+  for (int s = 0; s < kMaxPartialSplits; ++s)
+    t[s] = ldcg4_if(base + (size_t)s * sp.bn * 128, s < sp.k_splits);
   float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
-  for (int s = 0; s < sp.k_splits; ++s) {
-    const float4 t = __ldcg(reinterpret_cast<const float4*>(base + (size_t)s * sp.bn * 128));
-    a.x += t.x;
-    a.y += t.y;
-    a.z += t.z;
-    a.w += t.w;
+#pragma unroll
+  for (int s = 0; s < kMaxPartialSplits; ++s) {
+    if (s < sp.k_splits) {
+      a.x += t[s].x;
+      a.y += t[s].y;
+      a.z += t[s].z;
+      a.w += t[s].w;
+    }
   }
   bf16* dst;
   if (hs < Hq + Hkv) {

@@ -50,7 +50,7 @@ JF_DEV uint8_t* align1024(uint8_t* p) {
 // ---------------------------------------------------------------------------------------------
 template <typename T, int EPI>
 JF_DEV void epilogue_chunk(const GemmEpi& e, const float (&v)[16], int row, int n0, int m0, int c0, float* xs,
-                           int n_tile, int n_tiles) {
+                           int n_tile, int slot, int n_slots) {
   const int n = n0 + row;
   constexpr int kind = EPI;
   if constexpr (kind == EPI_STORE || kind == EPI_RESID) {
@@ -163,42 +163,88 @@ JF_DEV void epilogue_chunk(const GemmEpi& e, const float (&v)[16], int row, int 
         else { b2 = fmaxf(b2, o1); }
       }
       if (m < e.M) {
-        const size_t at = (size_t)m * n_tiles + n_tile;
-        e.am_v1[at] = b1;
-        e.am_i1[at] = bi;
-        e.am_v2[at] = b2;
+        // fold this tile into the CTA's running (best, index, runner-up) of row m; the same
+        // thread owns the slot for every tile of the CTA, so program order orders the updates
+        const size_t at = (size_t)m * n_slots + slot;
+        const float o1 = e.am_v1[at], o2 = e.am_v2[at];
+        const int oi = e.am_i1[at];
+        if (better(b1, bi, o1, oi)) {
+          e.am_v1[at] = b1;
+          e.am_i1[at] = bi;
+          e.am_v2[at] = fmaxf(o1, b2);
+        } else {
+          e.am_v2[at] = fmaxf(o2, b1);
+        }
       }
     }
     epi_sync();
   }
 }
 
-// Last CTA of a token tile: reduce the per-tile argmax partials of rows m0..m0+BN-1.
-JF_DEV void argmax_finish(const GemmEpi& e, int m0, int BN, int n_tiles, int tid) {
+// Argmax partials: slot (m, s) holds CTA s's running (best value, its index, runner-up value) of
+// row m over the vocabulary tiles that CTA has folded in. Every CTA starts its slots empty.
+JF_DEV void argmax_init_slots(const GemmEpi& e, int m_begin, int m_end, int slot, int n_slots, int tid, int nthreads) {
+  if (m_end > e.M) m_end = e.M;
+  for (int m = m_begin + tid; m < m_end; m += nthreads) {
+    const size_t at = (size_t)m * n_slots + slot;
+    e.am_v1[at] = -INFINITY;
+    e.am_i1[at] = 0x7fffffff;
+    e.am_v2[at] = -INFINITY;
+  }
+}
+
+JF_DEV void am_merge(float& b1, int& bi, float& b2, float o1, int oi, float o2) {
+  if (better(o1, oi, b1, bi)) { b2 = fmaxf(b1, o2); b1 = o1; bi = oi; }
+  else { b2 = fmaxf(b2, o1); }
+}
+
+// Last CTA of a token tile: reduce the slots of rows m0..m0+BN-1. Warp w takes rows two at a
+// time, lane l the slots l, l+32, ...; each round issues all loads of 2 rows x 4 slots per lane
+// before the first merge. The merge is associative and commutative, so the result does
+// not depend on which CTA folded which tile.
+constexpr int kAmSlotLoads = 4;  // slots per lane in flight per round
+JF_DEV void argmax_finish(const GemmEpi& e, int m0, int BN, int n_slots, int tid) {
   const int warp = tid >> 5, lane = tid & 31;
-  for (int r = warp; r < BN; r += 4) {
-    const int m = m0 + r;
-    if (m >= e.M) break;
-    float b1 = -INFINITY, b2 = -INFINITY;
-    int bi = 0x7fffffff;
-    for (int t = lane; t < n_tiles; t += 32) {
-      const size_t at = (size_t)m * n_tiles + t;
-      const float o1 = __ldcg(e.am_v1 + at), o2 = __ldcg(e.am_v2 + at);
-      const int oi = __ldcg(e.am_i1 + at);
-      if (better(o1, oi, b1, bi)) { b2 = fmaxf(b1, o2); b1 = o1; bi = oi; }
-      else { b2 = fmaxf(b2, o1); }
+  for (int r0 = warp * 2; r0 < BN; r0 += 8) {
+    float b1[2] = {-INFINITY, -INFINITY}, b2[2] = {-INFINITY, -INFINITY};
+    int bi[2] = {0x7fffffff, 0x7fffffff};
+    for (int s0 = 0; s0 < n_slots; s0 += 32 * kAmSlotLoads) {
+      float v1[2][kAmSlotLoads], v2[2][kAmSlotLoads];
+      int i1[2][kAmSlotLoads];
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        const int m = m0 + r0 + q;
+#pragma unroll
+        for (int k = 0; k < kAmSlotLoads; ++k) {
+          const int s = s0 + lane + 32 * k;
+          const bool ok = (r0 + q < BN) && m < e.M && s < n_slots;
+          const size_t at = (size_t)(ok ? m : 0) * n_slots + (ok ? s : 0);
+          v1[q][k] = ok ? __ldcg(e.am_v1 + at) : -INFINITY;
+          i1[q][k] = ok ? __ldcg(e.am_i1 + at) : 0x7fffffff;
+          v2[q][k] = ok ? __ldcg(e.am_v2 + at) : -INFINITY;
+        }
+      }
+#pragma unroll
+      for (int q = 0; q < 2; ++q)
+#pragma unroll
+        for (int k = 0; k < kAmSlotLoads; ++k) am_merge(b1[q], bi[q], b2[q], v1[q][k], i1[q][k], v2[q][k]);
     }
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float o1 = __shfl_xor_sync(0xffffffffu, b1, o);
-      const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-      const float o2 = __shfl_xor_sync(0xffffffffu, b2, o);
-      if (better(o1, oi, b1, bi)) { b2 = fmaxf(b1, o2); b1 = o1; bi = oi; }
-      else { b2 = fmaxf(b2, o1); }
-    }
-    if (lane == 0) {
-      e.am_out[m] = bi;
-      if (e.top2_out) { e.top2_out[2 * m] = b1; e.top2_out[2 * m + 1] = b2; }
+    for (int q = 0; q < 2; ++q) {
+      const int m = m0 + r0 + q;
+      float b1q = b1[q], b2q = b2[q];
+      int biq = bi[q];
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const float o1 = __shfl_xor_sync(0xffffffffu, b1q, o);
+        const int oi = __shfl_xor_sync(0xffffffffu, biq, o);
+        const float o2 = __shfl_xor_sync(0xffffffffu, b2q, o);
+        am_merge(b1q, biq, b2q, o1, oi, o2);
+      }
+      if (lane == 0 && r0 + q < BN && m < e.M) {
+        e.am_out[m] = biq;
+        if (e.top2_out) { e.top2_out[2 * m] = b1q; e.top2_out[2 * m + 1] = b2q; }
+      }
     }
   }
 }
@@ -238,7 +284,7 @@ JF_DEV void finish_tile_epi(const GemmParams& p, Get get, float* xs, int* sflag,
     for (int c = 0; c < nchunks; ++c) {
       float v[16];
       get(c * 16, v);
-      epilogue_chunk<T, EPI>(p.epi, v, tid, n0, m0, c * 16, xs, n_tile, p.n_tiles);
+      epilogue_chunk<T, EPI>(p.epi, v, tid, n0, m0, c * 16, xs, n_tile, blockIdx.x, gridDim.x);
     }
   } else {
     float* mine = p.ws + ((size_t)tile_lin * p.k_splits + split) * (size_t)BN * kTileN;
@@ -279,7 +325,7 @@ JF_DEV void finish_tile_epi(const GemmParams& p, Get get, float* xs, int* sflag,
           for (int j = 0; j < 16; ++j) v[j] += part[s][j];
         }
       }
-      epilogue_chunk<T, EPI>(p.epi, v, tid, n0, m0, c * 16, xs, n_tile, p.n_tiles);
+      epilogue_chunk<T, EPI>(p.epi, v, tid, n0, m0, c * 16, xs, n_tile, blockIdx.x, gridDim.x);
     }
     if (tid == 0) p.tile_counter[tile_lin] = 0;
   }
@@ -295,7 +341,7 @@ JF_DEV void finish_tile_epi(const GemmParams& p, Get get, float* xs, int* sflag,
     epi_sync();
     if (last) {
       __threadfence();
-      argmax_finish(p.epi, m0, BN, p.n_tiles, tid);
+      argmax_finish(p.epi, m0, BN, gridDim.x, tid);
       if (tid == 0) p.epi.am_counter[m_tile] = 0;
     }
   }
@@ -347,6 +393,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + S);
   const uint32_t tfull0 = smem_u32(bars + 2 * S), tempty0 = smem_u32(bars + 2 * S + 2);
   const int total_units = p.n_tiles * p.m_tiles * p.k_splits;
+  // The next kernel may launch as soon as every CTA of this grid is resident: its CTAs take the
+  // SMs this grid leaves, prefetch their own weights and park in their dependency wait, so no
+  // launch latency is paid after the last tile (it writes nothing before that wait).
+  pdl_launch_dependents();
 
   // producer: initialise the barriers, then request the first weight stages right away (weights do
   // not depend on earlier kernels, so they stream in while the previous kernel finishes)
@@ -469,6 +519,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   } else {
     // epilogue warps 0-3
     pdl_wait();
+    if constexpr (EPI == EPI_ARGMAX) {
+      argmax_init_slots(p.epi, 0, p.M, blockIdx.x, gridDim.x, tid, 128);
+      epi_sync();
+    }
     const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
     int i = 0;
     for (int u = blockIdx.x; u < total_units; u += gridDim.x, ++i) {
@@ -487,7 +541,6 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       if (tid == 0) mbar_arrive(tempty0 + 8 * acc);
     }
   }
-  pdl_launch_dependents();
   tc_fence_before();
   __syncthreads();
   if (warp == 4) tmem_dealloc(tmem, Cfg::TMEM_COLS);
@@ -542,6 +595,10 @@ __global__ void __launch_bounds__(128) k_gemm_f32(const float* __restrict__ W, c
         for (int j = 0; j < 16; ++j) v[j] = acc[cc + j];
       }
   };
+  if constexpr (EPI == EPI_ARGMAX) {
+    argmax_init_slots(p.epi, m0, m0 + F32_BN, blockIdx.x, gridDim.x, tid, 128);
+    __syncthreads();
+  }
   finish_tile<float, F32_BN, EPI>(p, get, xs, &sflag, blockIdx.x, 0, blockIdx.z, tid);
 }
 

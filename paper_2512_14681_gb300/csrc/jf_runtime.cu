@@ -38,6 +38,7 @@ using namespace jf;
 namespace {
 
 constexpr int kTargetCTAs = 152;   // split-K target: about one CTA per SM of a GB300
+constexpr int kMaxGemmGrid = 256;  // persistent GEMM grids (one CTA per SM) never exceed this
 // kernel classes of jf_kernel_time (include/jf.h)
 enum ProfClass : int {
   PC_GATEUP = 0, PC_ATTN = 1, PC_GEMMS = 2, PC_QKV = 3, PC_OPROJ = 4, PC_DOWN = 5, PC_LMHEAD = 6, PC_COMBINE = 7,
@@ -214,9 +215,9 @@ Offsets plan_offsets(const Dims& D) {
   o.gemm_ws = p.take(std::max<size_t>(o.gemm_ws_bytes, 16), 1024);
   const int max_mt = cdiv(D.R, 16) + 1;
   o.gemm_counter = p.take((size_t)(D.n_vtiles + 8) * max_mt * 4 + (size_t)(cdiv(2 * D.F, kTileN) + 8) * max_mt * 4);
-  o.am_v1 = p.take((size_t)D.R * D.n_vtiles * 4);
-  o.am_i1 = p.take((size_t)D.R * D.n_vtiles * 4);
-  o.am_v2 = p.take((size_t)D.R * D.n_vtiles * 4);
+  o.am_v1 = p.take((size_t)D.R * std::max(D.n_vtiles, kMaxGemmGrid) * 4);  // [row][CTA slot]
+  o.am_i1 = p.take((size_t)D.R * std::max(D.n_vtiles, kMaxGemmGrid) * 4);  // [row][CTA slot]
+  o.am_v2 = p.take((size_t)D.R * std::max(D.n_vtiles, kMaxGemmGrid) * 4);  // [row][CTA slot]
   o.am_counter = p.take((size_t)max_mt * 4);
   o.logits = p.take((size_t)std::max(D.logits_rows, 1) * D.V * 4, 1024);
   o.err = p.take(16);
@@ -883,6 +884,7 @@ jf_status jf_create(const jf_model_config* model, const jf_runtime_config* rt, j
   c->base = reinterpret_cast<char*>(rup(reinterpret_cast<uintptr_t>(rt->device_arena), 1024));
   cudaGetDevice(&c->device);
   cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device);
+  c->num_sms = std::min(c->num_sms, kMaxGemmGrid);
   if (rt->cuda_stream) {
     c->st = reinterpret_cast<cudaStream_t>(rt->cuda_stream);
   } else {

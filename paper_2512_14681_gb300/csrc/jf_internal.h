@@ -26,6 +26,7 @@ constexpr int kAttnQRows = 128;   // (token, head) query rows per attention work
 constexpr int kAttnLanes = 8;     // chunk lanes per unit (c mod 8); one CTA of an 8-CTA cluster each
 constexpr int kAttnLaneChunks = 128;  // chunks per lane the kernel can stage page ids for
 constexpr int kAttnMaxCtx = kAttnChunk * kAttnLanes * kAttnLaneChunks;  // 131072 key positions
+constexpr int kAttnXchgFloats = kAttnQRows * 128 + 2 * kAttnQRows;   // one lane state: O (hd 128), m, l
 constexpr int kMaxSeqs = 64;
 constexpr int kMaxChains = 256;
 
@@ -107,6 +108,7 @@ struct AttnParams {
   int Hq, Hkv, hd;
   float scale_log2;     // log2(e) / sqrt(hd)
   int* err;
+  float* xchg;          // bf16 path: lane states [unit][lane][kAttnXchgFloats]
 };
 
 // Host-side launch helpers (jf_kernels.cu). All launches use programmatic dependent launch.

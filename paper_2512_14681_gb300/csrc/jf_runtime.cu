@@ -26,9 +26,8 @@ cudaError_t launch_rmsnorm(float* x, const float* gain, void* y, bool is_bf16, i
                            const SplitPartials* acc, int row0, cudaStream_t st);
 cudaError_t launch_qkv_finish(const SplitPartials& sp, const int* pos, const float2* rope, void* q, void* k, void* v,
                               int M, int Hq, int Hkv, cudaStream_t st);
-cudaError_t launch_attn_bf16(const AttnParams& a, int units_bound, cudaStream_t st);
+cudaError_t launch_attn_tc(const AttnParams& a, int units_bound, cudaStream_t st);
 cudaError_t launch_attn_f32(const AttnParams& a, int n_rows, cudaStream_t st);
-size_t attn_bf16_smem_bytes();
 cudaError_t gemm_prepare();
 cudaError_t attn_prepare();
 }  // namespace jf
@@ -110,7 +109,7 @@ struct Offsets {
   std::vector<size_t> w_qkv, w_o, w_gu, w_d, g_attn, g_mlp;
   size_t k_pages, v_pages, page_table, seq_len, commit;
   size_t k_inf, v_inf, x, h, q, att, act;
-  size_t tok, pos, gpred, top2, chains, n_chains;
+  size_t tok, pos, gpred, top2, chains, n_chains, attn_xchg;
   size_t gemm_ws, gemm_counter, am_v1, am_i1, am_v2, am_counter;
   size_t logits, err;
   size_t gen_state, gen_out, gen_truth, gen_log, gen_q0, gen_plast, res, step_blocks, step_res, committed;
@@ -211,6 +210,8 @@ Offsets plan_offsets(const Dims& D) {
   o.top2 = p.take((size_t)D.R * 8);
   o.chains = p.take((size_t)kMaxChains * sizeof(Chain));
   o.n_chains = p.take(16);
+  // attention lane states: [unit][lane][128 x 128 O, 128 m, 128 l] fp32 (bf16 path)
+  o.attn_xchg = p.take(D.bf16 ? (size_t)D.max_units * kAttnLanes * kAttnXchgFloats * 4 : 16, 1024);
   o.gemm_ws_bytes = gemm_ws_floats(D) * 4;
   o.gemm_ws = p.take(std::max<size_t>(o.gemm_ws_bytes, 16), 1024);
   const int max_mt = cdiv(D.R, 16) + 1;
@@ -284,6 +285,7 @@ struct jf_ctx {
   float* top2;
   Chain* chains;
   int* n_chains;
+  float* attn_xchg;
   int chains_bound = 1;  // most chains the next forward can have (sizes the attention launch)
   float* gemm_ws;
   int* gemm_counter;
@@ -509,11 +511,12 @@ cudaError_t enqueue_forward(jf_ctx* c, int M, LmMode lm) {
     a.out = c->att; a.Hq = D.Hq; a.Hkv = D.Hkv; a.hd = D.hd;
     a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)D.hd));
     a.err = c->err;
+    a.xchg = c->attn_xchg;
     prof_begin(c, PC_ATTN);
     if (D.bf16) {
       // units of this forward are bounded by its rows: every chain adds at most one partial tile
       const int units_bound = std::min(D.max_units, D.Hkv * (cdiv((long long)M * D.G, kAttnQRows) + c->chains_bound));
-      e = launch_attn_bf16(a, units_bound, c->st);
+      e = launch_attn_tc(a, units_bound, c->st);
       prof_end(c);
     } else {
       e = launch_attn_f32(a, M, c->st);
@@ -928,6 +931,7 @@ jf_status jf_create(const jf_model_config* model, const jf_runtime_config* rt, j
   c->gpred = at<int>(c, O.gpred);
   c->top2 = at<float>(c, O.top2);
   c->chains = at<Chain>(c, O.chains);
+  c->attn_xchg = at<float>(c, O.attn_xchg);
   c->n_chains = at<int>(c, O.n_chains);
   c->gemm_ws = at<float>(c, O.gemm_ws);
   c->gemm_counter = at<int>(c, O.gemm_counter);

@@ -77,11 +77,27 @@ JF_DEV void epilogue_chunk(const GemmEpi& e, const float (&v)[16], int row, int 
       }
     }
     return;
-  } else if constexpr (kind == EPI_QKV || kind == EPI_SWIGLU) {
+  } else if constexpr (kind == EPI_SWIGLU) {
+    // rows 2i (gate) and 2i+1 (up) of the tile are feature 64 * n_tile + i, held by adjacent lanes:
+    // the even lane finishes columns 0..7 of the chunk, the odd lane columns 8..15
+    const bool odd = (row & 1) != 0;
+    const int f = n_tile * 64 + (row >> 1);
+    T* act = reinterpret_cast<T*>(e.act);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const float mine = odd ? v[k] : v[8 + k];
+      const float other = __shfl_xor_sync(0xffffffffu, mine, 1);
+      const float g = odd ? other : v[k];
+      const float u = odd ? v[8 + k] : other;
+      const int m = m0 + c0 + (odd ? 8 + k : k);
+      if (m < e.M && n < e.N) act[(size_t)m * e.ld_act + f] = to_act<T>(silu_f(g) * u);
+    }
+    return;
+  } else if constexpr (kind == EPI_QKV) {
 #pragma unroll
     for (int j = 0; j < 16; ++j) xs[j * 128 + row] = v[j];
     epi_sync();
-    if constexpr (kind == EPI_QKV) {
+    {
       const int hd = e.head_dim, half = hd >> 1;
       const int i = n % hd;
       const bool is_q = n < e.n_q;
@@ -113,16 +129,6 @@ JF_DEV void epilogue_chunk(const GemmEpi& e, const float (&v)[16], int row, int 
             out = (i < half) ? (out * cs[j].x - x2 * cs[j].y) : (out * cs[j].x + x2 * cs[j].y);
           }
           if (m < e.M) dst[(size_t)m * stride] = to_act<T>(out);
-        }
-      }
-    } else {
-      if (row < 64) {
-        const int f = n_tile * 64 + row;
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {
-          const int m = m0 + c0 + j;
-          const float g = xs[j * 128 + row], u = xs[j * 128 + row + 64];
-          if (m < e.M) reinterpret_cast<T*>(e.act)[(size_t)m * e.ld_act + f] = to_act<T>(silu_f(g) * u);
         }
       }
     }

@@ -70,7 +70,7 @@ struct GemmEpi {
   int n_q, n_kv, head_dim;
   const int* pos;
   const float2* rope;   // [max_pos][hd/2] (cos, sin)
-  // EPI_SWIGLU: tile t holds gate rows 64t..64t+63 then the matching up rows; act[m][64t + i]
+  // EPI_SWIGLU: tile t holds features 64t..64t+63 as row pairs (gate 64t+i at 2i, up at 2i+1); act[m][64t + i]
   void* act;
   int ld_act;
   // EPI_ARGMAX: per (row, tile) partial (v1, i1, v2), ticket per token tile, final argmax/top2

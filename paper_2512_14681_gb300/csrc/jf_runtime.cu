@@ -267,6 +267,7 @@ struct jf_ctx {
   bool own_stream = false;
   int device = 0;
   int num_sms = 152;
+  int o_splits = 0;   // split-K of the O projection (0: from the weight shape; never above it)
   std::string last_error;
   bool weights_ready = false;
   // device pointers
@@ -431,7 +432,7 @@ void prof_end(jf_ctx* c) {
 }
 
 cudaError_t gemm(jf_ctx* c, const CUtensorMap& tmA, const void* W, const void* X, int N, int K, int M,
-                 const GemmEpi& epi, int cls) {
+                 const GemmEpi& epi, int cls, int splits = 0) {
   const Dims& D = c->D;
   GemmParams p;
   p.N = N; p.K = K; p.M = M;
@@ -450,7 +451,7 @@ cudaError_t gemm(jf_ctx* c, const CUtensorMap& tmA, const void* W, const void* X
   if (D.bf16) {
     const int bn = gemm_bn_for(M);
     p.m_tiles = cdiv(M, bn);
-    p.k_splits = splits_for(p.n_tiles, p.kb_total);
+    p.k_splits = splits > 0 ? std::min(splits, splits_for(p.n_tiles, p.kb_total)) : splits_for(p.n_tiles, p.kb_total);
     CUtensorMap tmB;
     if (!make_tmap(&tmB, X, K, M, bn)) return cudaErrorInvalidValue;
     e = launch_gemm_bf16(tmA, tmB, p, bn, c->st);
@@ -477,11 +478,13 @@ cudaError_t enqueue_forward(jf_ctx* c, int M, LmMode lm) {
   // the following RMSNorms add them (split order) instead of a last-CTA reduction in the GEMM
   const bool partials = D.bf16;
   const bool qkv_partial = partials && D.hd == kTileN;
-  auto split_parts = [&](int N, int K) {
+  auto split_parts = [&](int N, int K, int splits) {
     const int bn = gemm_bn_for(M);
-    return SplitPartials{c->gemm_ws, splits_for(cdiv(N, kTileN), cdiv(K, kTileK)), cdiv(M, bn), bn};
+    const int auto_sp = splits_for(cdiv(N, kTileN), cdiv(K, kTileK));
+    return SplitPartials{c->gemm_ws, splits > 0 ? std::min(splits, auto_sp) : auto_sp, cdiv(M, bn), bn};
   };
-  const SplitPartials sp_qkv = split_parts(D.nqkv, D.d), sp_o = split_parts(D.d, D.nq), sp_dn = split_parts(D.d, D.F);
+  const SplitPartials sp_qkv = split_parts(D.nqkv, D.d, 0), sp_o = split_parts(D.d, D.nq, c->o_splits),
+                      sp_dn = split_parts(D.d, D.F, 0);
   for (int l = 0; l < D.L; ++l) {
     LayerW& w = c->layers[l];
     char* kinf = reinterpret_cast<char*>(c->k_inf) + l * inf_layer;
@@ -525,7 +528,7 @@ cudaError_t enqueue_forward(jf_ctx* c, int M, LmMode lm) {
     if (e != cudaSuccess) return e;
     GemmEpi er = {};
     er.kind = partials ? EPI_PARTIAL : EPI_RESID; er.x = c->x; er.ldx = D.d;
-    if ((e = gemm(c, w.tm_o, w.o, c->att, D.d, D.nq, M, er, PC_OPROJ)) != cudaSuccess) return e;
+    if ((e = gemm(c, w.tm_o, w.o, c->att, D.d, D.nq, M, er, PC_OPROJ, c->o_splits)) != cudaSuccess) return e;
     prof_begin(c, PC_NORM);
     e = launch_rmsnorm(c->x, w.g_mlp, c->h, D.bf16, M, D.d, eps, partials ? &sp_o : nullptr, 0, c->st);
     prof_end(c);
@@ -1026,8 +1029,8 @@ bool tensor_loc(jf_ctx* c, int tid, TensorLoc* t) {
     case 3: t->base = (char*)L.qkv; t->rows = D.nkv; t->cols = D.d; t->grp_off = D.nq + D.nkv; return true;
     case 4: t->base = (char*)L.o; t->rows = D.d; t->cols = D.nq; return true;
     case 5: t->base = (char*)L.g_mlp; t->rows = 1; t->cols = D.d; t->gain = true; return true;
-    case 6: t->base = (char*)L.gu; t->rows = D.F; t->cols = D.d; t->grp = 64; t->grp_stride = 128; return true;
-    case 7: t->base = (char*)L.gu; t->rows = D.F; t->cols = D.d; t->grp = 64; t->grp_stride = 128; t->grp_off = 64; return true;
+    case 6: t->base = (char*)L.gu; t->rows = D.F; t->cols = D.d; t->grp = 1; t->grp_stride = 2; return true;
+    case 7: t->base = (char*)L.gu; t->rows = D.F; t->cols = D.d; t->grp = 1; t->grp_stride = 2; t->grp_off = 1; return true;
     case 8: t->base = (char*)L.dn; t->rows = D.d; t->cols = D.F; return true;
   }
   return false;
@@ -1041,6 +1044,26 @@ std::vector<int> all_tids(const Dims& D) {
 }
 
 long long dev_row(const TensorLoc& t, long long r) { return (r / t.grp) * t.grp_stride + (r % t.grp) + t.grp_off; }
+
+// Whole tensor between its device rows and a dense host buffer [rows][cols]: one strided 2-D copy
+// of the full groups of t.grp rows, one more for a partial last group.
+cudaError_t copy_tensor(const TensorLoc& t, int es, void* host, cudaMemcpyKind kind) {
+  const size_t rb = (size_t)t.cols * es;
+  const bool to_dev = kind == cudaMemcpyHostToDevice;
+  if (t.grp >= t.rows) {
+    char* dev = t.base + (size_t)t.grp_off * rb;
+    return to_dev ? cudaMemcpy(dev, host, (size_t)t.rows * rb, kind) : cudaMemcpy(host, dev, (size_t)t.rows * rb, kind);
+  }
+  const long long full = t.rows / t.grp, tail = t.rows % t.grp;
+  const size_t gw = (size_t)t.grp * rb, dp = (size_t)t.grp_stride * rb;
+  char* h = reinterpret_cast<char*>(host);
+  char* dev = t.base + (size_t)t.grp_off * rb;
+  cudaError_t e = to_dev ? cudaMemcpy2D(dev, dp, h, gw, gw, (size_t)full, kind) : cudaMemcpy2D(h, gw, dev, dp, gw, (size_t)full, kind);
+  if (e != cudaSuccess || tail == 0) return e;
+  char* dt = t.base + (size_t)dev_row(t, full * t.grp) * rb;
+  char* ht = h + (size_t)full * gw;
+  return to_dev ? cudaMemcpy(dt, ht, (size_t)tail * rb, kind) : cudaMemcpy(ht, dt, (size_t)tail * rb, kind);
+}
 
 struct FileHeader {
   char magic[4];
@@ -1112,20 +1135,17 @@ jf_status jf_save_weights(jf_ctx* c, const char* path) {
                   c->mc.head_dim, c->mc.d_ff, c->mc.vocab, c->mc.rms_eps, c->mc.rope_theta};
   bool ok = std::fwrite(&h, sizeof(h), 1, f) == 1;
   CK(cudaStreamSynchronize(c->st));
-  std::vector<uint8_t> row;
+  std::vector<uint8_t> buf;
   for (int tid : all_tids(c->D)) {
     TensorLoc t;
     tensor_loc(c, tid, &t);
     const int es = t.gain ? 4 : c->D.es;
-    row.resize((size_t)t.cols * es);
-    for (long long r = 0; r < t.rows && ok; ++r) {
-      if (cudaMemcpy(row.data(), t.base + (size_t)dev_row(t, r) * t.cols * es, row.size(), cudaMemcpyDeviceToHost) !=
-          cudaSuccess) {
-        std::fclose(f);
-        return fail(c, JF_ECUDA, "copy of weights failed");
-      }
-      ok = std::fwrite(row.data(), 1, row.size(), f) == row.size();
+    buf.resize((size_t)t.rows * t.cols * es);
+    if (copy_tensor(t, es, buf.data(), cudaMemcpyDeviceToHost) != cudaSuccess) {
+      std::fclose(f);
+      return fail(c, JF_ECUDA, "copy of weights failed");
     }
+    ok = ok && std::fwrite(buf.data(), 1, buf.size(), f) == buf.size();
   }
   ok = (std::fclose(f) == 0) && ok;
   return ok ? JF_OK : fail(c, JF_EIO, "short write of weight file");
@@ -1165,16 +1185,7 @@ jf_status jf_load_weights(jf_ctx* c, const char* path) {
   for (size_t i = 0; i < locs.size(); ++i) {
     const TensorLoc& t = locs[i];
     const int es = t.gain ? 4 : c->D.es;
-    const size_t rb = (size_t)t.cols * es;
-    if (t.grp >= t.rows) {
-      CK(cudaMemcpy(t.base + (size_t)t.grp_off * rb, data[i].data(), data[i].size(), cudaMemcpyHostToDevice));
-    } else {
-      for (long long r0 = 0; r0 < t.rows; r0 += t.grp) {
-        const long long n = std::min(t.grp, t.rows - r0);
-        CK(cudaMemcpy(t.base + (size_t)dev_row(t, r0) * rb, data[i].data() + (size_t)r0 * rb, (size_t)n * rb,
-                      cudaMemcpyHostToDevice));
-      }
-    }
+    CK(copy_tensor(t, es, data[i].data(), cudaMemcpyHostToDevice));
   }
   c->weights_ready = true;
   return JF_OK;

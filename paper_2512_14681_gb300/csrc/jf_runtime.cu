@@ -267,7 +267,6 @@ struct jf_ctx {
   bool own_stream = false;
   int device = 0;
   int num_sms = 152;
-  int o_splits = 0;   // split-K of the O projection (0: from the weight shape; never above it)
   std::string last_error;
   bool weights_ready = false;
   // device pointers
@@ -432,7 +431,7 @@ void prof_end(jf_ctx* c) {
 }
 
 cudaError_t gemm(jf_ctx* c, const CUtensorMap& tmA, const void* W, const void* X, int N, int K, int M,
-                 const GemmEpi& epi, int cls, int splits = 0) {
+                 const GemmEpi& epi, int cls) {
   const Dims& D = c->D;
   GemmParams p;
   p.N = N; p.K = K; p.M = M;
@@ -451,7 +450,7 @@ cudaError_t gemm(jf_ctx* c, const CUtensorMap& tmA, const void* W, const void* X
   if (D.bf16) {
     const int bn = gemm_bn_for(M);
     p.m_tiles = cdiv(M, bn);
-    p.k_splits = splits > 0 ? std::min(splits, splits_for(p.n_tiles, p.kb_total)) : splits_for(p.n_tiles, p.kb_total);
+    p.k_splits = splits_for(p.n_tiles, p.kb_total);
     CUtensorMap tmB;
     if (!make_tmap(&tmB, X, K, M, bn)) return cudaErrorInvalidValue;
     e = launch_gemm_bf16(tmA, tmB, p, bn, c->st);
@@ -478,13 +477,11 @@ cudaError_t enqueue_forward(jf_ctx* c, int M, LmMode lm) {
   // the following RMSNorms add them (split order) instead of a last-CTA reduction in the GEMM
   const bool partials = D.bf16;
   const bool qkv_partial = partials && D.hd == kTileN;
-  auto split_parts = [&](int N, int K, int splits) {
+  auto split_parts = [&](int N, int K) {
     const int bn = gemm_bn_for(M);
-    const int auto_sp = splits_for(cdiv(N, kTileN), cdiv(K, kTileK));
-    return SplitPartials{c->gemm_ws, splits > 0 ? std::min(splits, auto_sp) : auto_sp, cdiv(M, bn), bn};
+    return SplitPartials{c->gemm_ws, splits_for(cdiv(N, kTileN), cdiv(K, kTileK)), cdiv(M, bn), bn};
   };
-  const SplitPartials sp_qkv = split_parts(D.nqkv, D.d, 0), sp_o = split_parts(D.d, D.nq, c->o_splits),
-                      sp_dn = split_parts(D.d, D.F, 0);
+  const SplitPartials sp_qkv = split_parts(D.nqkv, D.d), sp_o = split_parts(D.d, D.nq), sp_dn = split_parts(D.d, D.F);
   for (int l = 0; l < D.L; ++l) {
     LayerW& w = c->layers[l];
     char* kinf = reinterpret_cast<char*>(c->k_inf) + l * inf_layer;
@@ -528,7 +525,7 @@ cudaError_t enqueue_forward(jf_ctx* c, int M, LmMode lm) {
     if (e != cudaSuccess) return e;
     GemmEpi er = {};
     er.kind = partials ? EPI_PARTIAL : EPI_RESID; er.x = c->x; er.ldx = D.d;
-    if ((e = gemm(c, w.tm_o, w.o, c->att, D.d, D.nq, M, er, PC_OPROJ, c->o_splits)) != cudaSuccess) return e;
+    if ((e = gemm(c, w.tm_o, w.o, c->att, D.d, D.nq, M, er, PC_OPROJ)) != cudaSuccess) return e;
     prof_begin(c, PC_NORM);
     e = launch_rmsnorm(c->x, w.g_mlp, c->h, D.bf16, M, D.d, eps, partials ? &sp_o : nullptr, 0, c->st);
     prof_end(c);

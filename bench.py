@@ -46,6 +46,7 @@ class Workload:
     pool: int = 0       # rejection-recycling pool entries
     ngram: int = 0      # n-gram length (0 = n)
     cands: int = 0      # recycled candidates verified per iteration
+    spawn: float = 0.0  # spawn ratio r: a new block starts once the newest has ceil(r n) accepted tokens
 
 
 # The 7B single-block workload at p = 0.3 is the headline; the others are the remaining decode
@@ -62,13 +63,18 @@ WORKLOADS = {w.name: w for w in [
              "qwen2.5-1.5b-shape-bf16", 512, 16, 256, 0.5),
     Workload("qwen2.5-7b-shape-bf16 prompt2048 blocks4x32 rr-pool64x32 cand1 new1024 inject-p0.3 paged-kv16 bs1",
              "qwen2.5-7b-shape-bf16", 2048, 32, 1024, 0.3, blocks=4, pool=64, ngram=32, cands=1),
+    # the paper's inference configuration for its method (Sec. 4.3 / App. E): K = 2 blocks of n = 64,
+    # spawn ratio r = 0.85, 4 recycled n-grams verified per iteration (up to 384 rows in flight)
+    Workload("qwen2.5-7b-shape-bf16 prompt1024 blocks2x64 spawn0.85 rr-pool64x64 cand4 new512 inject-p0.3 paged-kv16 bs1",
+             "qwen2.5-7b-shape-bf16", 1024, 64, 512, 0.3, blocks=2, pool=64, ngram=64, cands=4, spawn=0.85),
 ]}
 DEFAULT_WORKLOAD = next(iter(WORKLOADS))
 ALIASES = {"7b": DEFAULT_WORKLOAD, "7b-p0.1": list(WORKLOADS)[1], "7b-p0.7": list(WORKLOADS)[2],
-           "1.5b": list(WORKLOADS)[3], "7b-mb4-rr": list(WORKLOADS)[4]}
-# DRAM bytes (read + write) per launch of the gate/up projection at M = 32 rows, from the ncu capture
-# summarised in profiles/gateup_gemm_7b_m32.md; None until a capture of the current kernel exists.
-GATEUP_TRAFFIC_BYTES = None
+           "1.5b": list(WORKLOADS)[3], "7b-mb4-rr": list(WORKLOADS)[4], "7b-mr-k2n64": list(WORKLOADS)[5]}
+# DRAM bytes (read + write) per launch of the gate/up projection at M = 32 rows: dram__bytes_read.sum
+# + dram__bytes_write.sum of one `ncu --set full` capture of the current kernel (271.90 MB weights
+# and activations read, 3.64 MB SwiGLU output written). Set to None whenever the kernel changes.
+GATEUP_TRAFFIC_BYTES = 275_537_152
 
 
 def _peaks():
@@ -230,8 +236,8 @@ def run_gpu(args, rank, world, local_rank):
     ctx.init_random_weights(I.WEIGHT_SEED, I.WEIGHT_STD)
     prompt = I.prompt_tokens(shape.vocab, PROMPT_LEN)
     truth = ctx.generate([prompt], Gen(mode="ar", max_new=truth_len)).tokens[0].astype(np.int32)
-    gen = Gen(block_size=BLOCK, n_blocks=wl.blocks, pool_size=wl.pool, ngram_len=wl.ngram, cand_per_iter=wl.cands,
-              init="inject", inject_p=P_INJECT, seed=I.INJECT_SEED, max_new=NEW)
+    gen = Gen(block_size=BLOCK, n_blocks=wl.blocks, spawn_ratio=wl.spawn, pool_size=wl.pool, ngram_len=wl.ngram,
+              cand_per_iter=wl.cands, init="inject", inject_p=P_INJECT, seed=I.INJECT_SEED, max_new=NEW)
     d_prompt = torch.from_numpy(prompt).cuda()
     d_truth = torch.from_numpy(truth).cuda().reshape(1, -1)
     d_out = torch.empty((1, NEW), dtype=torch.int32, device="cuda")
@@ -324,7 +330,8 @@ def run_gpu(args, rank, world, local_rank):
                 "greedy continuation",
         "config": {"workload": args.workload if not args.layers else f"{args.workload} ({args.layers}-layer profiling case)",
                    "layers": shape.n_layers, "prompt": PROMPT_LEN, "block_size": BLOCK, "new_tokens": NEW,
-                   "blocks": wl.blocks, "rr_pool": wl.pool, "ngram": G, "candidates": wl.cands,
+                   "blocks": wl.blocks, "spawn_ratio": wl.spawn, "rr_pool": wl.pool, "ngram": G,
+                   "candidates": wl.cands,
                    "rows_per_iteration_max": rows_per_iter,
                    "inject_p": P_INJECT, "kv_page_tokens": 16, "batch": 1,
                    "parallelism": "replicas" if world > 1 else "single-gpu",

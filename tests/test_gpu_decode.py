@@ -29,6 +29,9 @@ MODES = {
     "inj_window": dict(block_size=8, mode="window", init="inject", inject_p=0.3, seed=2),
     "inj_block": dict(block_size=8, init="inject", inject_p=0.5, seed=3),
     "inj_mb_rr": dict(block_size=8, n_blocks=4, pool_size=16, cand_per_iter=1, init="inject", inject_p=0.3, seed=4),
+    # the shape of the paper's inference configuration (K = 2, r = 0.85, 4 verified n-grams), small n
+    "inj_mr_k2_r085_c4": dict(block_size=8, n_blocks=2, spawn_ratio=0.85, pool_size=16, cand_per_iter=4,
+                              init="inject", inject_p=0.3, seed=5),
 }
 
 

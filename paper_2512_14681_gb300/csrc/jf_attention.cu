@@ -46,8 +46,15 @@ JF_DEV void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uin
                : "r"(addr));
 }
 JF_DEV uint32_t pack_bf16(float lo, float hi) {
-  const bf16 l = __float2bfloat16_rn(lo), h = __float2bfloat16_rn(hi);
-  return (uint32_t)__bfloat16_as_ushort(l) | ((uint32_t)__bfloat16_as_ushort(h) << 16);
+  const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);  // one cvt.rn.bf16x2.f32
+  return *reinterpret_cast<const uint32_t*>(&v);
+}
+
+// 2^x by the MUFU ex2 instruction (flushes results below 2^-126 to zero; 2^-inf = 0).
+JF_DEV float ex2_ftz(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
 }
 
 // Fold of two softmax states (m, l, O) in the log2 domain: m = max(ma, mb),
@@ -302,27 +309,31 @@ __global__ void __maxnreg__(200) k_attn_tc(const AttnParams a) {
       for (int i = 0; i < 32; ++i) sv[32 + i] = t32[i];
     }
     const int kbase = sub_of(t) * kAttnChunk + 64 * half;
+    // mask (key position <= row position) on the raw scores; the scale (> 0) goes into the row
+    // maximum and into one fma per exponential: p = 2^(s * scale - m)
+    const float scale = a.scale_log2;
     float mx = -INFINITY;
 #pragma unroll
     for (int i = 0; i < 64; ++i) {
-      sv[i] = (kbase + i <= pos_r) ? sv[i] * a.scale_log2 : -INFINITY;
+      sv[i] = (kbase + i <= pos_r) ? sv[i] : -INFINITY;
       mx = fmaxf(mx, sv[i]);
     }
-    red_max[half][r] = mx;
+    red_max[half][r] = mx * scale;
     ok = __syncthreads_and(ok) != 0;  // keeps the loop's barriers uniform across the CTA
     const float mn = fmaxf(m_run, fmaxf(red_max[0][r], red_max[1][r]));
-    const float al = (m_run == -INFINITY) ? 0.f : exp2f(m_run - mn);
-    const float b = (mn == -INFINITY) ? 0.f : mn;
+    const float al = (m_run == -INFINITY) ? 0.f : ex2_ftz(m_run - mn);
+    const float nb = (mn == -INFINITY) ? 0.f : -mn;
     m_run = mn;
-    l_run *= al;
-    // P (bf16) into this stage's K block `half` (S is complete, K is no longer read)
+    // P (bf16) into this stage's K block `half` (S is complete, K is no longer read); the row sum
+    // in four independent partial sums, added in a fixed order
+    float ls[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
     for (int c = 0; c < 8; ++c) {
       float p[8];
 #pragma unroll
       for (int e = 0; e < 8; ++e) {
-        p[e] = exp2f(sv[8 * c + e] - b);
-        l_run += p[e];
+        p[e] = ex2_ftz(fmaf(sv[8 * c + e], scale, nb));
+        ls[e & 3] += p[e];
       }
       const uint4 w = make_uint4(pack_bf16(p[0], p[1]), pack_bf16(p[2], p[3]), pack_bf16(p[4], p[5]),
                                  pack_bf16(p[6], p[7]));
@@ -330,6 +341,7 @@ __global__ void __maxnreg__(200) k_attn_tc(const AttnParams a) {
       asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(dst), "r"(w.x), "r"(w.y), "r"(w.z), "r"(w.w)
                    : "memory");
     }
+    l_run = l_run * al + ((ls[0] + ls[1]) + (ls[2] + ls[3]));
     fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();

@@ -80,15 +80,15 @@ __global__ void k_embed(const T* __restrict__ E, const int* __restrict__ tok, fl
 }
 
 // y[r, :] = x[r, :] / sqrt(mean(x[r, :]^2) + eps) * gain, rounded to the activation type.
-// One CTA of 512 threads per row; the row stays in registers (float4, up to 4 per thread:
+// One CTA of 1024 threads per row; the row stays in registers (float4, up to 2 per thread:
 // d <= 8192), so x is read once. The reduction order is fixed by d alone.
 // ACC: the residual update of the preceding projection is finished here first: the k_splits
 // partial sums of x's increment (EPI_PARTIAL) are added in split order, x += that sum is written
 // back, and the norm is taken of the updated row. Every load of a row is issued before the first
 // add (the row's bytes are one round trip), which is what bounds this kernel. Rows are
 // row0 + blockIdx.x.
-constexpr int NORM_THREADS = 512;
-constexpr int NORM_VEC = 4;
+constexpr int NORM_THREADS = 1024;
+constexpr int NORM_VEC = 2;
 constexpr int kMaxPartialSplits = 8;  // the host never splits K more than this
 
 // L2-cached 16-byte load that yields zeros when `pred` is false. Volatile: a run of these is
@@ -103,6 +103,25 @@ __device__ __forceinline__ float4 ldcg4_if(const float* p, bool pred) {
   return v;
 }
 
+// Four L2-cached 16-byte loads p, p + stride, p + 2 stride, p + 3 stride (floats) in one asm
+// statement: all four are issued before any of their results is used; load k is skipped (zeros)
+// when k >= n.
+__device__ __forceinline__ void ldcg4x4(const float* p, size_t stride, int n, float4 (&q)[4]) {
+#pragma unroll
+  for (int k = 0; k < 4; ++k) q[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+  asm volatile(
+      "{\n\t.reg .pred p0, p1, p2, p3;\n\t"
+      "setp.gt.s32 p0, %20, 0;\n\tsetp.gt.s32 p1, %20, 1;\n\tsetp.gt.s32 p2, %20, 2;\n\tsetp.gt.s32 p3, %20, 3;\n\t"
+      "@p0 ld.global.cg.v4.f32 {%0,%1,%2,%3}, [%16];\n\t"
+      "@p1 ld.global.cg.v4.f32 {%4,%5,%6,%7}, [%17];\n\t"
+      "@p2 ld.global.cg.v4.f32 {%8,%9,%10,%11}, [%18];\n\t"
+      "@p3 ld.global.cg.v4.f32 {%12,%13,%14,%15}, [%19];\n\t}"
+      : "+f"(q[0].x), "+f"(q[0].y), "+f"(q[0].z), "+f"(q[0].w), "+f"(q[1].x), "+f"(q[1].y), "+f"(q[1].z), "+f"(q[1].w),
+        "+f"(q[2].x), "+f"(q[2].y), "+f"(q[2].z), "+f"(q[2].w), "+f"(q[3].x), "+f"(q[3].y), "+f"(q[3].z), "+f"(q[3].w)
+      : "l"(p), "l"(p + stride), "l"(p + 2 * stride), "l"(p + 3 * stride), "r"(n)
+      : "memory");
+}
+
 __device__ __forceinline__ void store4(float* y, float4 v) { *reinterpret_cast<float4*>(y) = v; }
 __device__ __forceinline__ void store4(bf16* y, float4 v) {
   const uint32_t lo = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.x)) |
@@ -112,7 +131,7 @@ __device__ __forceinline__ void store4(bf16* y, float4 v) {
   *reinterpret_cast<uint2*>(y) = make_uint2(lo, hi);
 }
 
-template <typename T, bool ACC>
+template <typename T, int KS>
 __global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(float* __restrict__ x, const float* __restrict__ gain,
                                                           T* __restrict__ y, int d, float eps, SplitPartials sp,
                                                           int row0) {
@@ -128,40 +147,31 @@ __global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(float* __restrict__ x,
     const int i = threadIdx.x + j * NORM_THREADS;
     v[j] = (i < nv) ? xr[i] : make_float4(0.f, 0.f, 0.f, 0.f);
   }
-  if constexpr (ACC) {
-    // two vectors' partials (and the row itself, above) in flight together
+  if constexpr (KS > 0) {
+    // the KS split partials of a vector: KS independent loads, then added in split order
 #pragma unroll
-    for (int j0 = 0; j0 < NORM_VEC; j0 += 2) {
-      if (j0 * NORM_THREADS >= nv) break;
-      float4 q[2][kMaxPartialSplits];
-#pragma unroll
-      for (int jj = 0; jj < 2; ++jj) {
-        const int i = threadIdx.x + (j0 + jj) * NORM_THREADS;
+    for (int j = 0; j < NORM_VEC; ++j) {
+      if (j * NORM_THREADS >= nv) break;
+      const int i = threadIdx.x + j * NORM_THREADS;
+      if (i < nv) {
         const int n = 4 * i;
-        const float* base = sp.ws + ((size_t)((n >> 7) * sp.m_tiles + r / sp.bn) * sp.k_splits * sp.bn +
+        const float* base = sp.ws + ((size_t)((n >> 7) * sp.m_tiles + r / sp.bn) * KS * sp.bn +
                                      (size_t)(r % sp.bn)) * 128 + (n & 127);
+        constexpr int NB = (KS + 3) / 4;
+        float4 q[NB][4];
+        const size_t stride = (size_t)sp.bn * 128;
 #pragma unroll
-        for (int s = 0; s < kMaxPartialSplits; ++s)
-          q[jj][s] = ldcg4_if(base + (size_t)s * sp.bn * 128, i < nv && s < sp.k_splits);
-      }
+        for (int b = 0; b < NB; ++b) ldcg4x4(base + (size_t)(4 * b) * stride, stride, KS - 4 * b, q[b]);
+        float4 acc = q[0][0];
 #pragma unroll
-      for (int jj = 0; jj < 2; ++jj) {
-        const int i = threadIdx.x + (j0 + jj) * NORM_THREADS;
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-        for (int s = 0; s < kMaxPartialSplits; ++s) {
-          if (s < sp.k_splits) {
-            acc.x += q[jj][s].x;
-            acc.y += q[jj][s].y;
-            acc.z += q[jj][s].z;
-            acc.w += q[jj][s].w;
-          }
+        for (int s = 1; s < KS; ++s) {
+          acc.x += q[s >> 2][s & 3].x;
+          acc.y += q[s >> 2][s & 3].y;
+          acc.z += q[s >> 2][s & 3].z;
+          acc.w += q[s >> 2][s & 3].w;
         }
-        const int j = j0 + jj;
-        if (i < nv) {
-          v[j] = make_float4(v[j].x + acc.x, v[j].y + acc.y, v[j].z + acc.z, v[j].w + acc.w);
-          xr[i] = v[j];
-        }
+        v[j] = make_float4(v[j].x + acc.x, v[j].y + acc.y, v[j].z + acc.z, v[j].w + acc.w);
+        xr[i] = v[j];
       }
     }
   }
@@ -300,18 +310,32 @@ cudaError_t launch_embed(const void* E, bool is_bf16, const int* tok, float* x, 
   return launch_pdl(k_embed<float>, dim3(rows), dim3(256), st, reinterpret_cast<const float*>(E), tok, x, d, V, err);
 }
 
+template <int KS>
+cudaError_t launch_rmsnorm_ks(float* x, const float* gain, bf16* y, int rows, int d, float eps,
+                              const SplitPartials& sp, int row0, cudaStream_t st) {
+  return launch_pdl(k_rmsnorm<bf16, KS>, dim3(rows), dim3(NORM_THREADS), st, x, gain, y, d, eps, sp, row0);
+}
+
 cudaError_t launch_rmsnorm(float* x, const float* gain, void* y, bool is_bf16, int rows, int d, float eps,
                            const SplitPartials* acc, int row0, cudaStream_t st) {
   const SplitPartials sp = acc ? *acc : SplitPartials{nullptr, 0, 1, 1};
   if (is_bf16) {
-    if (acc)
-      return launch_pdl(k_rmsnorm<bf16, true>, dim3(rows), dim3(NORM_THREADS), st, x, gain, reinterpret_cast<bf16*>(y),
-                        d, eps, sp, row0);
-    return launch_pdl(k_rmsnorm<bf16, false>, dim3(rows), dim3(NORM_THREADS), st, x, gain, reinterpret_cast<bf16*>(y),
-                      d, eps, sp, row0);
+    bf16* yb = reinterpret_cast<bf16*>(y);
+    switch (acc ? sp.k_splits : 0) {
+      case 0: return launch_rmsnorm_ks<0>(x, gain, yb, rows, d, eps, sp, row0, st);
+      case 1: return launch_rmsnorm_ks<1>(x, gain, yb, rows, d, eps, sp, row0, st);
+      case 2: return launch_rmsnorm_ks<2>(x, gain, yb, rows, d, eps, sp, row0, st);
+      case 3: return launch_rmsnorm_ks<3>(x, gain, yb, rows, d, eps, sp, row0, st);
+      case 4: return launch_rmsnorm_ks<4>(x, gain, yb, rows, d, eps, sp, row0, st);
+      case 5: return launch_rmsnorm_ks<5>(x, gain, yb, rows, d, eps, sp, row0, st);
+      case 6: return launch_rmsnorm_ks<6>(x, gain, yb, rows, d, eps, sp, row0, st);
+      case 7: return launch_rmsnorm_ks<7>(x, gain, yb, rows, d, eps, sp, row0, st);
+      case 8: return launch_rmsnorm_ks<8>(x, gain, yb, rows, d, eps, sp, row0, st);
+      default: return cudaErrorInvalidValue;
+    }
   }
   if (acc) return cudaErrorInvalidValue;
-  return launch_pdl(k_rmsnorm<float, false>, dim3(rows), dim3(NORM_THREADS), st, x, gain, reinterpret_cast<float*>(y),
+  return launch_pdl(k_rmsnorm<float, 0>, dim3(rows), dim3(NORM_THREADS), st, x, gain, reinterpret_cast<float*>(y),
                     d, eps, sp, row0);
 }
 

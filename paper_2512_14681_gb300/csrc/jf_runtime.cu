@@ -40,7 +40,7 @@ constexpr int kTargetCTAs = 152;   // split-K target: about one CTA per SM of a 
 constexpr int kMaxGemmGrid = 256;  // persistent GEMM grids (one CTA per SM) never exceed this
 // kernel classes of jf_kernel_time (include/jf.h)
 enum ProfClass : int {
-  PC_GATEUP = 0, PC_ATTN = 1, PC_GEMMS = 2, PC_QKV = 3, PC_OPROJ = 4, PC_DOWN = 5, PC_LMHEAD = 6, PC_COMBINE = 7,
+  PC_GATEUP = 0, PC_ATTN = 1, PC_GEMMS = 2, PC_QKV = 3, PC_OPROJ = 4, PC_DOWN = 5, PC_LMHEAD = 6, PC_RESERVED = 7,
   PC_NORM = 8, PC_OTHER = 9, kProfClasses = 10
 };
 constexpr int kMaxStateInts = 32768;

@@ -166,3 +166,30 @@ def test_short_prompt_and_short_generation(tiny):
     ar = J.generate_ar(tiny, p, 5)
     res = J.generate_jacobi(tiny, p, J.GenParams(block_size=8, max_new=5))
     assert res.tokens == ar.tokens and len(res.tokens) == 5
+
+
+@pytest.mark.parametrize("init", ["repeat", "inject"])
+def test_paper_inference_configuration_is_lossless(tiny, prompt, ar64, init):
+    """K = 2 blocks, spawn ratio r = 0.85, 4 recycled n-grams verified per iteration (the paper's
+    chosen configuration, Sec. 4.3), at a small block size: still exactly the AR greedy output."""
+    # injection needs the truth beyond max_new (K n + G + 1 more tokens than are generated)
+    max_new = 39 if init == "inject" else 64
+    kw = dict(block_size=8, n_blocks=2, spawn_ratio=0.85, pool_size=16, cand_per_iter=4, max_new=max_new)
+    if init == "inject":
+        kw.update(init="inject", inject_p=0.3, seed=5)
+    res = J.generate_jacobi(tiny, prompt, J.GenParams(**kw), truth=ar64.tokens if init == "inject" else None)
+    assert res.tokens == ar64.tokens[:max_new]
+
+
+def test_second_block_spawns_at_the_threshold(tiny, prompt, ar64):
+    """Algorithm 1: the next block starts once the newest one holds ceil(r n) accepted tokens.
+    With p = 0 injection every draft is exact, so the first block commits all n = 8 tokens in its
+    first iteration; with r = 0.85 (threshold 7) the second block spawns right after it, never
+    before. Before the spawn the forward carries only the first block's rows."""
+    res = J.generate_jacobi(tiny, prompt, J.GenParams(block_size=8, n_blocks=2, spawn_ratio=0.85, init="inject",
+                                                      inject_p=0.0, seed=1, max_new=32), truth=ar64.tokens)
+    assert res.tokens == ar64.tokens[:32]
+    assert res.iters[0].M == 8 and res.iters[0].k == 8 and res.iters[0].pseudo == []
+    # a ratio of 0 (threshold 0) has both blocks in flight from the first iteration
+    eager = J.generate_jacobi(tiny, prompt, J.GenParams(block_size=8, n_blocks=2, spawn_ratio=0.0, max_new=16))
+    assert eager.iters[0].M == 16 and len(eager.iters[0].pseudo) == 1

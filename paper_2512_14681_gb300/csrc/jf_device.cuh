@@ -71,7 +71,7 @@ JF_DEV bool mbar_wait_bounded(uint32_t bar, uint32_t parity, uint64_t limit_ns) 
 constexpr uint64_t JF_WAIT_LIMIT_NS = 2000000000ull;  // 2 s: far beyond any legitimate wait
 
 // ------------------------------------------------------------------------------------------
-// Thread-block clusters: ranks, cluster-wide barrier, distributed shared memory
+// Thread-block clusters: ranks, cluster-wide barrier
 // ------------------------------------------------------------------------------------------
 JF_DEV uint32_t cluster_rank() {
   uint32_t r;
@@ -86,67 +86,6 @@ JF_DEV uint32_t cluster_id_x() {
 JF_DEV void cluster_sync() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
-// Split cluster barrier: arrive (release) early, wait (acquire) later.
-JF_DEV void cluster_arrive() { asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory"); }
-JF_DEV void cluster_wait() { asm volatile("barrier.cluster.wait.aligned;" ::: "memory"); }
-JF_DEV uint32_t dsmem_addr(uint32_t local, uint32_t rank) {
-  uint32_t r;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local), "r"(rank));
-  return r;
-}
-JF_DEV float dsmem_ld_f32(uint32_t addr) {
-  float v;
-  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr) : "memory");
-  return v;
-}
-JF_DEV void dsmem_st_f32(uint32_t addr, float v) {
-  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(addr), "f"(v) : "memory");
-}
-JF_DEV void dsmem_st_f32x2(uint32_t addr, float a, float b) {
-  asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(addr), "f"(a), "f"(b) : "memory");
-}
-JF_DEV void dsmem_st_f32x4(uint32_t addr, float4 v) {
-  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w)
-               : "memory");
-}
-JF_DEV float4 dsmem_ld_f32x4(uint32_t addr) {
-  float4 v;
-  asm volatile("ld.shared::cluster.v4.f32 {%0,%1,%2,%3}, [%4];"
-               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-               : "r"(addr)
-               : "memory");
-  return v;
-}
-
-// Bulk copy of `bytes` (multiple of 16, both addresses 16-byte aligned) from this CTA's shared
-// memory to shared::cluster address `dst`, completing transaction bytes on the mbarrier at
-// shared::cluster address `mbar` (in the destination CTA).
-JF_DEV void bulk_copy_to_cluster(uint32_t dst, uint32_t src, uint32_t bytes, uint32_t mbar) {
-  asm volatile("cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
-               "r"(src), "r"(bytes), "r"(mbar)
-               : "memory");
-}
-JF_DEV bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-// Wait (acquire, cluster scope) for phase `parity` of a local mbarrier that peers complete.
-JF_DEV bool mbar_wait_cluster_bounded(uint32_t bar, uint32_t parity, uint64_t limit_ns) {
-  if (mbar_try_wait_cluster(bar, parity)) return true;
-  const uint64_t t0 = jf_globaltimer();
-  while (true) {
-    if (mbar_try_wait_cluster(bar, parity)) return true;
-    if (jf_globaltimer() - t0 > limit_ns) return false;
-  }
-}
-
 // ------------------------------------------------------------------------------------------
 // TMA (cp.async.bulk.tensor) loads with an L2 cache-policy hint
 // ------------------------------------------------------------------------------------------

@@ -37,7 +37,7 @@ struct Chain {
   int seq, row0, nrows, pos0;
 };
 
-// Attention work unit: (chain, KV head, tile of 64 (token, head) query rows), its chain resolved;
+// Attention work unit: (chain, KV head, tile of 128 (token, head) query rows), its chain resolved;
 // `pad` is nonzero for a unit that exists.
 struct AttnUnit {
   int seq, row0, nrows, pos0, kvh, qt, n_chunks, pad;
@@ -73,7 +73,8 @@ struct GemmEpi {
   // EPI_SWIGLU: tile t holds features 64t..64t+63 as row pairs (gate 64t+i at 2i, up at 2i+1); act[m][64t + i]
   void* act;
   int ld_act;
-  // EPI_ARGMAX: per (row, tile) partial (v1, i1, v2), ticket per token tile, final argmax/top2
+  // EPI_ARGMAX: per (row, CTA) running (v1, i1, v2) slot, one ticket per token tile; the CTA that
+  // completes a token tile folds the slots into the final argmax / top-2
   float* am_v1;
   int* am_i1;
   float* am_v2;
@@ -86,7 +87,7 @@ struct GemmParams {
   int N, K, M;
   int n_tiles, m_tiles, k_splits, kb_total;
   int grid;            // persistent CTAs (bf16 path): at most one per SM
-  float* ws;           // split-K partials [m_tiles*n_tiles][k_splits][BN][128]
+  float* ws;           // split-K partials [n_tiles][m_tiles][k_splits][BN][128]
   int* tile_counter;   // [m_tiles*n_tiles], zero between launches
   int* err;
   GemmEpi epi;
@@ -111,7 +112,8 @@ struct AttnParams {
   float* xchg;          // bf16 path: lane states [unit][lane][kAttnXchgFloats]
 };
 
-// Host-side launch helpers (jf_kernels.cu). All launches use programmatic dependent launch.
+// Host-side launch helpers of the projection GEMM (jf_gemm.cu) and the TMA descriptor encoder
+// (jf_runtime.cu). All launches use programmatic dependent launch.
 cudaError_t launch_gemm_bf16(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmParams& p, int bn,
                              cudaStream_t st);
 cudaError_t launch_gemm_f32(const float* W, const float* X, const GemmParams& p, cudaStream_t st);

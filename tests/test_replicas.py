@@ -35,7 +35,7 @@ def _worker(rank, world, port, out):
 def test_replica_throughput_is_total_tokens_over_slowest_rank():
     world = 2
     port = _free_port()
-    mgr = mp.Manager()
+    mgr = mp.get_context("spawn").Manager()  # no fork of this (threaded) test process
     out = mgr.dict()
     mp.spawn(_worker, args=(world, port, out), nprocs=world, join=True)
     for r in range(world):

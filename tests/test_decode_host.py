@@ -1,0 +1,200 @@
+"""The CUDA decoding state machine (csrc/jf_decode.cu: verification, pool, pseudo-accept, tail update,
+spawn / promote, next rows and chains; Algorithm 1, Sec. 3.2, Eq. 3-4) compiled for the CPU and
+checked without a GPU (tests/decode_host/build.py says how the kernels become host code).
+
+* Against the hand-derived traces of tests/golden/ (toy predictor, scripted drafts).
+* Its draft-injection rule against the oracle's, on many (seed, position, iteration) keys.
+* Against the oracle's decoding loop under the same toy predictor on randomised configurations
+  (blocks, spawn ratio, pool, candidates, n-gram length, window mode, batch, injection rate,
+  EOS): rows, committed counts, winners and tokens of every iteration must agree.
+"""
+import ctypes
+import glob
+import math
+import os
+import shutil
+import types
+
+import numpy as np
+import pytest
+
+from oracle import jacobi as J
+from tests.toy_decode import chain_predictions, parse, toy_module, wrong_const
+
+pytestmark = pytest.mark.skipif(shutil.which("g++") is None, reason="needs g++")
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+CASES = [c for c in sorted(glob.glob(os.path.join(GOLDEN, "*.txt"))) if not c.endswith("README.txt")]
+
+
+@pytest.fixture(scope="module")
+def hd():
+    from tests.decode_host import build as HB
+
+    return HB.load()
+
+
+def _p(a):
+    return a.ctypes.data_as(ctypes.POINTER(ctypes.c_int))
+
+
+def run_device(hd, pr, prompts, truths, stationary, V, script=None, wrong=wrong_const):
+    """Drive the host-compiled state machine with toy predictions. Returns per sequence the list of
+    its iterations (rows M, committed count k, winner, output tokens) and its generated tokens."""
+    ns = len(prompts)
+    if pr.mode == "ar":
+        n, K, mode, pool, C = 1, 1, 1, 0, 0
+    else:
+        n, K, mode, pool = pr.block_size, pr.n_blocks, (1 if pr.mode == "window" else 0), pr.pool_size
+        C = pr.cand_per_iter if pool > 0 else 0
+    G = pr.ngram_len or n
+    init = 1 if pr.init == "inject" else 0
+    s_spawn = math.ceil(pr.spawn_ratio * n - 1e-12)
+    T = int(float(np.float32(pr.inject_p)) * 2**53)
+    truth_len = min(len(t) - len(p) for t, p in zip(truths, prompts)) if init else 0
+    assert not init or truth_len >= pr.max_new + K * n + G + 1
+    truth_arr = np.zeros((ns, max(truth_len, 1)), dtype=np.int32)
+    for b in range(ns):
+        if init:
+            truth_arr[b] = truths[b][len(prompts[b]):len(prompts[b]) + truth_len]
+    max_rows = ns * (K * n + C * G)
+    max_chains = ns * (1 + C)
+    max_ctx = max(len(p) for p in prompts) + pr.max_new + K * n + G + 8
+    assert hd.hd_setup(n, K, s_spawn, pool, G, C, mode, init, T, pr.seed, pr.max_new, pr.eos_id, V, ns,
+                       _p(truth_arr), truth_len, max_rows, max_chains, max_ctx) == 0
+    if script is None:
+        hd.hd_script(-1, None, None, None)
+    else:
+        ks = sorted(script)
+        cols = [np.array(c, dtype=np.int32) for c in ([k[0] for k in ks], [k[1] for k in ks], [script[k] for k in ks])]
+        hd.hd_script(len(ks), *[_p(c) for c in cols])
+    committed = [list(p) for p in prompts]
+    q0 = np.array([truths[b][len(prompts[b])] for b in range(ns)], dtype=np.int32)  # the toy's prefill argmax
+    seq_len = np.array([len(p) for p in prompts], dtype=np.int32)
+    plast = np.array([p[-1] for p in prompts], dtype=np.int32)
+    hd.hd_init(_p(q0), _p(seq_len), _p(plast))
+    tok = np.zeros(max_rows, dtype=np.int32)
+    pos = np.zeros(max_rows, dtype=np.int32)
+    ch = np.zeros((max_chains, 4), dtype=np.int32)
+    hdr = np.zeros(4, dtype=np.int32)
+    k, win, nout, P = (np.zeros(ns, dtype=np.int32) for _ in range(4))
+    cm = np.zeros((ns, 3), dtype=np.int32)
+    out = np.zeros((ns, pr.max_new), dtype=np.int32)
+    recs = [[] for _ in range(ns)]
+
+    def view():
+        hd.hd_view(_p(tok), _p(pos), _p(ch), _p(hdr), _p(k), _p(win), _p(nout), _p(P), _p(cm))
+        assert hdr[3] == 0, f"device error word {hdr[3]}"
+
+    view()
+    done = [False] * ns
+    for _ in range(4 * (pr.max_new + 4)):
+        if hdr[2]:
+            break
+        M = int(hdr[0])
+        chains = [tuple(int(v) for v in ch[c]) for c in range(int(hdr[1]))]
+        rows = [0] * ns
+        for s, _, nr, _ in chains:
+            rows[s] += nr
+        cur_tok = [int(t) for t in tok[:M]]
+        pred = np.array(chain_predictions(cur_tok, [int(x) for x in pos[:M]], chains, committed, truths, stationary,
+                                          wrong), dtype=np.int32)
+        prev_out = nout.copy()
+        hd.hd_accept(_p(pred), M)
+        view()
+        hd.hd_out_tokens(_p(out))
+        for b in range(ns):
+            if done[b]:
+                assert k[b] == 0 and rows[b] == 0
+                continue
+            row0, kk, p_at = (int(v) for v in cm[b])
+            assert p_at == len(committed[b]) and kk == k[b]
+            committed[b] += cur_tok[row0:row0 + kk]  # the rows the KV commit copies into the cache
+            recs[b].append(dict(M=rows[b], k=int(k[b]), winner=int(win[b]),
+                                out=[int(t) for t in out[b, prev_out[b]:nout[b]]]))
+            done[b] = bool(nout[b] >= pr.max_new or (pr.eos_id >= 0 and pr.eos_id in out[b, :nout[b]]))
+    else:
+        raise AssertionError("decoding did not terminate")
+    assert all(done)
+    return recs, [[int(t) for t in out[b, :nout[b]]] for b in range(ns)]
+
+
+def run_oracle(pr, prompt, truth_seq, stationary, V, monkeypatch, wrong=wrong_const):
+    toy = toy_module(truth_seq, stationary, wrong)
+    toy.sm64 = J.O.sm64  # the injection rule's generator stays the oracle's own
+    monkeypatch.setattr(J, "O", toy)
+    model = types.SimpleNamespace(cfg=types.SimpleNamespace(vocab=V))
+    truth = truth_seq[len(prompt):] if pr.init == "inject" else None
+    return J.JacobiDecoder(model, prompt, pr, truth=truth).run()
+
+
+@pytest.mark.parametrize("path", CASES, ids=[os.path.basename(c)[:-4] for c in CASES])
+def test_device_state_machine_matches_hand_derived_trace(hd, path):
+    spec = parse(path)
+    pr = J.GenParams(**spec["params"])
+    T = spec["prompt"] + spec["truth"]
+    recs, toks = run_device(hd, pr, [spec["prompt"]], [T], [spec["stationary"]], 1000, script=spec["corrupt"])
+    assert len(recs[0]) == len(spec["iters"])
+    for i, (have, want) in enumerate(zip(recs[0], spec["iters"])):
+        assert (have["M"], have["k"], have["winner"], have["out"]) == \
+            (want["M"], want["k"], want["winner"], want["committed"]), f"iteration {i}"
+    assert toks[0] == spec["tokens"]
+
+
+def test_device_injection_rule_equals_oracle(hd):
+    """The kernels' injection rule and the oracle's, each written from the SplitMix64 definition."""
+    rng = np.random.default_rng(5)
+    for _ in range(3000):
+        seed = int(rng.integers(0, 2**63))
+        p = float(rng.choice([0.0, 0.1, 0.3, 0.5, 0.7, 1.0]))
+        T = J.inject_threshold(p)
+        V = int(rng.choice([2, 3, 1000, 152064]))
+        truth_tok = int(rng.integers(0, V))
+        x, it = int(rng.integers(0, 1 << 20)), int(rng.integers(0, 4096))
+        assert hd.hd_inject_rule(seed, T, V, truth_tok, x, it) == J.inject_token(seed, x, it, truth_tok, T, V)
+
+
+def _random_case(rng):
+    mode = str(rng.choice(["block", "block", "block", "window", "ar"]))
+    n = int(rng.choice([1, 2, 3, 4, 6, 8]))
+    K = int(rng.integers(1, 4)) if mode == "block" else 1
+    pool = int(rng.choice([0, 0, 2, 4, 8]))
+    C = int(rng.integers(1, 4)) if pool else 0
+    G = int(rng.choice([0, 0, 2, 3, 5]))
+    init = str(rng.choice(["repeat", "inject"]))
+    return J.GenParams(block_size=n, n_blocks=K, spawn_ratio=float(rng.choice([0.0, 0.25, 0.5, 0.85, 1.0])),
+                       pool_size=pool, ngram_len=G, cand_per_iter=C, mode=mode, init=init,
+                       inject_p=float(rng.choice([0.0, 0.2, 0.5, 0.9])), seed=int(rng.integers(0, 1 << 30)),
+                       max_new=int(rng.integers(1, 40)), eos_id=-1)
+
+
+@pytest.mark.parametrize("case_seed", range(300))
+def test_device_state_machine_equals_oracle_loop(hd, case_seed, monkeypatch):
+    """Randomised configurations; a small vocabulary makes chance matches (lucky drafts, pool keys,
+    wrong predictions that agree) frequent, so rarely reached branches run."""
+    rng = np.random.default_rng(1000 + case_seed)
+    pr = _random_case(rng)
+    V = int(rng.choice([6, 12, 50]))
+    ns = int(rng.integers(1, 4))
+    eos = int(rng.integers(2, V)) if rng.random() < 0.25 else -1
+    pr = J.GenParams(**{**pr.__dict__, "eos_id": eos})
+    prompts, truths, stationary = [], [], []
+    for b in range(ns):
+        P0 = int(rng.integers(1, 6))
+        length = P0 + pr.max_new + pr.n_blocks * pr.block_size + (pr.ngram_len or pr.block_size) + 8
+        T = [int(t) for t in rng.integers(2, V, size=length)]
+        prompts.append(T[:P0])
+        truths.append(T)
+        stationary.append({int(x) for x in rng.integers(0, length, size=int(rng.integers(0, length // 3 + 1)))})
+    shift = int(rng.integers(0, V))
+
+    def wrong(x, t):
+        return (3 * t + x + shift) % V
+
+    recs, toks = run_device(hd, pr, prompts, truths, stationary, V, wrong=wrong)
+    for b in range(ns):
+        want = run_oracle(pr, prompts[b], truths[b], stationary[b], V, monkeypatch, wrong)
+        assert toks[b] == want.tokens, f"sequence {b}: {pr}"
+        assert len(recs[b]) == len(want.iters), f"sequence {b}: {pr}"
+        for i, (have, it) in enumerate(zip(recs[b], want.iters)):
+            assert (have["M"], have["k"], have["winner"]) == (it.M, it.k, it.winner), f"seq {b} iteration {i}: {pr}"

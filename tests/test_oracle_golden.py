@@ -1,6 +1,6 @@
 """The oracle's decoding loop (Algorithm 1, Sec. 3.2; Eq. 3-4) against hand-derived traces (no GPU).
 
-The transformer is replaced by a scripted toy predictor (described in tests/golden/README.txt) and the
+The transformer is replaced by a scripted toy predictor (tests/toy_decode.py) and the
 draft injection by a scripted corruption list, so that every iteration's rows, accepted counts,
 pseudo-accepted counts, winner and committed tokens can be worked out by hand. The traces under
 tests/golden/ were derived that way from the rules; this test runs the oracle's loop on the same
@@ -9,103 +9,18 @@ prefix position by position, and the toy forward applies the tree mask as Sec. 3
 sees the committed cache, its own segment causally, and every ancestor segment).
 """
 import glob
+import inspect
 import os
+import sys
 import types
 
-import numpy as np
 import pytest
 
 from oracle import jacobi as J
+from tests.toy_decode import parse, toy_module
 
 GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
-WRONG = 1
 VOCAB = 1000
-
-
-def _ints(s):
-    return [int(t) for t in s.replace(",", " ").split()] if s.strip() else []
-
-
-def parse(path):
-    spec = {"iters": [], "corrupt": {}, "stationary": set()}
-    for raw in open(path):
-        line = raw.split("#", 1)[0].strip()
-        if not line:
-            continue
-        head, _, rest = line.partition(" ")
-        if head == "params":
-            kw = {}
-            for item in rest.split():
-                k, v = item.split("=")
-                kw[k] = v if k in ("mode", "init") else (float(v) if k == "spawn_ratio" else int(v))
-            spec["params"] = kw
-        elif head == "model":
-            k, _, v = rest.partition("=")
-            assert k == "stationary"
-            spec["stationary"] = set(_ints(v))
-        elif head in ("prompt", "truth", "tokens"):
-            spec[head] = _ints(rest)
-        elif head == "corrupt":
-            for item in rest.split():
-                at, tok = item.split("=")
-                pos, it = at.split("@")
-                spec["corrupt"][(int(pos), int(it))] = int(tok)
-        elif head == "iter":
-            rec = {}
-            for item in rest.split():
-                k, v = item.split("=")
-                rec[k] = _ints(v) if k in ("k_cand", "pseudo", "committed") else int(v)
-            spec["iters"].append(rec)
-        else:
-            raise ValueError(f"{path}: unknown line {line!r}")
-    return spec
-
-
-class ToyCache:
-    """Committed tokens of one sequence; commit() takes rows of the last forward, in order, and checks
-    that they extend the prefix position by position (the cache trim of Algorithm 1)."""
-
-    def __init__(self, model, max_ctx, max_rows):
-        self.toks = []
-        self.last = None
-
-    def __len__(self):
-        return len(self.toks)
-
-    def commit(self, rows):
-        tokens, pos = self.last
-        for r in list(rows):
-            assert pos[r] == len(self.toks), "committed row is not the next position"
-            self.toks.append(int(tokens[r]))
-
-
-def toy_module(T, stationary):
-    def forward(model, cache, tokens, pos, seg=None, anc=None, **_):
-        tokens = [int(t) for t in tokens]
-        pos = [int(p) for p in pos]
-        M = len(tokens)
-        seg = [0] * M if seg is None else [int(s) for s in seg]
-        anc = [0] * (max(seg) + 1) if anc is None else [int(a) for a in anc]
-        P = len(cache)
-        assert all(p >= P for p in pos), "an in-flight row overlaps the committed prefix"
-        pred = []
-        for i in range(M):
-            x = pos[i]
-            if x - 1 < 0:
-                prev_ok = True
-            elif x - 1 < P:
-                prev_ok = cache.toks[x - 1] == T[x - 1]
-            else:
-                seen = [j for j in range(M) if pos[j] == x - 1 and
-                        ((seg[j] == seg[i] and pos[j] <= x) or (seg[j] != seg[i] and (anc[seg[i]] >> seg[j]) & 1))]
-                assert len(seen) <= 1, "two visible rows at one position"
-                prev_ok = bool(seen) and tokens[seen[0]] == T[x - 1]
-            ok = tokens[i] == T[x] and prev_ok
-            pred.append(T[x + 1] if ok or (x + 1) in stationary else WRONG)
-        cache.last = (tokens, pos)
-        return types.SimpleNamespace(argmax=np.array(pred, dtype=np.int32), margin=np.ones(M))
-
-    return types.SimpleNamespace(forward=forward, Cache=ToyCache)
 
 
 CASES = sorted(glob.glob(os.path.join(GOLDEN, "*.txt")))
@@ -149,3 +64,50 @@ def test_golden_traces_are_lossless():
         assert spec["tokens"] == spec["truth"][: len(spec["tokens"])], path
         flat = [t for it in spec["iters"] for t in it["committed"]]
         assert flat == spec["tokens"], path
+
+
+# Plausible mistakes in the decoding loop, each planted (in memory, on the CPU) into a copy of the
+# oracle's loop; every one must fail at least one hand-derived trace.
+PLANTED = {
+    "pseudo-accept compares with the row at the position itself":
+        ("blk.q[pk] == main_pred(blk.start + na + pk)", "blk.q[pk] == main_pred(blk.start + na + pk + 1)"),
+    "pseudo blocks do not see the blocks before them":
+        ("anc = [0] + [(1 << b) - 1 for b in range(1, n_main_seg)]", "anc = [0] * n_main_seg"),
+    "candidates ignore the key":
+        ("order = [i for i in range(len(self.pool) - 1, -1, -1) if self.pool[i][0] == self.q0]", "order = []"),
+    "Jacobi update shifted by one row":
+        ("return g[row0 + r]", "return g[row0 + r + 1] if row0 + r + 1 < len(g) else g[row0 + r]"),
+    "ties go to the candidate": ("if kc > k:", "if kc >= k:"),
+    "pool entries padded with token 0": ("ent += [ent[-1]] * (self.G - len(ent))", "ent += [0] * (self.G - len(ent))"),
+    "spawn needs more than ceil(r n)": ("if progress < s:", "if progress <= s:"),
+    "promotion keeps the block's own first token": ("draft[0] = self.q0", "pass"),
+    "pseudo drafts redrawn with the current iteration":
+        ("blk.q = [self._inj(x, self.it + 1) for x in range(lo, hi)]",
+         "blk.q = [self._inj(x, self.it) for x in range(lo, hi)]"),
+    "spawned block repeats the last committed token":
+        ("prev_tok = (last.a + last.q)[-1]", "prev_tok = self._last_committed()"),
+    "q0 taken from the draft's rows when a candidate wins":
+        ("new_q0, new_q0_margin = g[row0 + k - 1], mg[row0 + k - 1]", "new_q0, new_q0_margin = g[k - 1], mg[k - 1]"),
+    "pool entry stops at the end of the real-active draft":
+        ("ent = main_tok[k_ra:k_ra + self.G]", "ent = list(ra.q[k_ra:k_ra + self.G])"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(PLANTED))
+def test_planted_mistake_fails_a_trace(name, monkeypatch):
+    a, b = PLANTED[name]
+    src = inspect.getsource(J)
+    assert src.count(a) == 1
+    mod = types.ModuleType("oracle.jacobi_planted")
+    mod.__package__ = "oracle"
+    monkeypatch.setitem(sys.modules, mod.__name__, mod)  # its dataclasses look their module up there
+    exec(compile(src.replace(a, b), J.__file__, "exec"), mod.__dict__)
+    monkeypatch.setattr(sys.modules[__name__], "J", mod)
+    caught = 0
+    for path in CASES:
+        with pytest.MonkeyPatch.context() as mp:
+            try:
+                test_decoding_loop_matches_hand_derived_trace(path, mp)
+            except AssertionError:
+                caught += 1
+    assert caught > 0, name

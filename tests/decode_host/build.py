@@ -81,6 +81,8 @@ def load():
     lib.hd_view.restype = None
     lib.hd_out_tokens.argtypes = [ip]
     lib.hd_out_tokens.restype = None
+    lib.hd_step.argtypes = [i32, ip, ip, i32, ip, ip, ip, ip, ip]
+    lib.hd_step.restype = None
     lib.hd_inject_rule.argtypes = [u64, u64, i32, i32, i32, i32]
     lib.hd_inject_rule.restype = i32
     return lib

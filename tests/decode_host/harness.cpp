@@ -121,6 +121,32 @@ void hd_out_tokens(int* out) {
   for (size_t i = 0; i < out_tokens.size(); ++i) out[i] = out_tokens[i];
 }
 
+// Step-mode verification (caller-supplied blocks of one sequence): counts[n_blocks], then
+// (winner, k, q0_next, err) in out4, the committed tokens in committed[k].
+void hd_step(int n_blocks, const int* kind, const int* len, int P, const int* tok_in, const int* gpred, int* counts,
+             int* out4, int* committed_out) {
+  jf::StepBlocks sb{};
+  sb.n_blocks = n_blocks;
+  sb.seq = 0;
+  sb.P = P;
+  int total = 0;
+  for (int b = 0; b < n_blocks; ++b) {
+    sb.kind[b] = kind[b];
+    sb.row0[b] = total;
+    sb.len[b] = len[b];
+    total += len[b];
+  }
+  std::vector<jf::CommitInfo> ci(1);
+  jf::StepResult r{};
+  int e = 0;
+  jf::k_step_accept(&sb, tok_in, gpred, committed_out, ci.data(), &r, &e);
+  for (int b = 0; b < n_blocks; ++b) counts[b] = r.counts[b];
+  out4[0] = r.winner;
+  out4[1] = r.k;
+  out4[2] = r.q0_next;
+  out4[3] = r.err;
+}
+
 // The kernels' draft-injection rule for one (seed, threshold, position, iteration, truth token).
 int hd_inject_rule(unsigned long long seed, unsigned long long T, int V, int truth_tok, int x, int it) {
   jf::GenCfg g{};

@@ -198,3 +198,36 @@ def test_device_state_machine_equals_oracle_loop(hd, case_seed, monkeypatch):
         assert len(recs[b]) == len(want.iters), f"sequence {b}: {pr}"
         for i, (have, it) in enumerate(zip(recs[b], want.iters)):
             assert (have["M"], have["k"], have["winner"]) == (it.M, it.k, it.winner), f"seq {b} iteration {i}: {pr}"
+
+
+def test_step_mode_verification(hd):
+    """Caller-supplied blocks (the step call): a real-active draft or candidate accepts 1 + the run of
+    tokens equal to the prediction of the row before them; a pseudo block, whose rows continue the
+    block before it, accepts the run from its first token against the prediction of that block's
+    last row; the largest count among the draft and the candidates wins, ties to the earlier block."""
+    rng = np.random.default_rng(11)
+    for _ in range(2000):
+        V = int(rng.integers(2, 5))
+        kinds = [0] + [1] * int(rng.integers(0, 3)) + [2] * int(rng.integers(0, 3))
+        lens = [int(rng.integers(1, 7)) for _ in kinds]
+        M = sum(lens)
+        tok = rng.integers(0, V, size=M).astype(np.int32)
+        pred = rng.integers(0, V, size=M).astype(np.int32)
+        counts = np.zeros(len(kinds), dtype=np.int32)
+        out4 = np.zeros(4, dtype=np.int32)
+        com = np.full(M, -7, dtype=np.int32)
+        kind_a, len_a = np.array(kinds, dtype=np.int32), np.array(lens, dtype=np.int32)
+        hd.hd_step(len(kinds), _p(kind_a), _p(len_a), 100, _p(tok), _p(pred), _p(counts), _p(out4), _p(com))
+        want, best, win, r0 = [], 0, -1, 0
+        for b, (kd, ln) in enumerate(zip(kinds, lens)):
+            c = 0 if kd == 1 else 1
+            while c < ln and tok[r0 + c] == pred[r0 + c - 1]:
+                c += 1
+            want.append(c)
+            if kd != 1 and c > best:
+                best, win, wr0 = c, b, r0
+            r0 += ln
+        assert list(counts) == want
+        assert (out4[0], out4[1], out4[3]) == (win, best, 0)
+        assert out4[2] == pred[wr0 + best - 1]
+        assert list(com[:best]) == list(tok[wr0:wr0 + best])

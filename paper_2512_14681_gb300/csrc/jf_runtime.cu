@@ -698,6 +698,16 @@ void accumulate_profile(jf_ctx* c, GraphRec* g) {
   }
 }
 
+// Timing events of one call; destroyed on every return path (an event still pending in the stream
+// is released once the device reaches it).
+struct CallEvents {
+  cudaEvent_t e[3] = {nullptr, nullptr, nullptr};
+  ~CallEvents() {
+    for (cudaEvent_t x : e)
+      if (x) cudaEventDestroy(x);
+  }
+};
+
 jf_status generate_impl(jf_ctx* c, int n_seqs, const int32_t* const* h_prompts, const int32_t* d_prompts,
                         const int32_t* prompt_lens, const jf_gen_params* gp, int32_t* h_out, int32_t* d_out,
                         jf_gen_stats* stats, bool device_io) {
@@ -759,10 +769,11 @@ jf_status generate_impl(jf_ctx* c, int n_seqs, const int32_t* const* h_prompts, 
     if (s != JF_OK) return s;
   }
   const long long launches0 = c->launches;
-  cudaEvent_t e0, e1, e2;
-  CK(cudaEventCreate(&e0));
-  CK(cudaEventCreate(&e1));
-  CK(cudaEventCreate(&e2));
+  CallEvents ev;  // released on every return path
+  CK(cudaEventCreate(&ev.e[0]));
+  CK(cudaEventCreate(&ev.e[1]));
+  CK(cudaEventCreate(&ev.e[2]));
+  const cudaEvent_t e0 = ev.e[0], e1 = ev.e[1], e2 = ev.e[2];
   CK(cudaEventRecord(e0, c->st));
   std::vector<int> q0(n_seqs), plast(n_seqs);
   long long off = 0;
@@ -847,9 +858,6 @@ jf_status generate_impl(jf_ctx* c, int n_seqs, const int32_t* const* h_prompts, 
     if (stats->rows)
       for (int i = 0; i < cap; ++i) stats->rows[i] = rows_log[i];
   }
-  cudaEventDestroy(e0);
-  cudaEventDestroy(e1);
-  cudaEventDestroy(e2);
   return JF_OK;
 }
 

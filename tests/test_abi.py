@@ -95,3 +95,36 @@ def test_op_gemm_validation_and_workspace(lib):
     # K not a multiple of 8 (16-byte TMA rows) and null pointers are refused before any launch
     assert lib.jf_op_gemm(J.JF_BF16, 16, 16, 16, 128, 60, 4, 0, 16, 1 << 20, 16, None) == J.JF_EINVAL
     assert lib.jf_op_gemm(J.JF_BF16, None, 16, 16, 128, 64, 4, 0, 16, 1 << 20, 16, None) == J.JF_EINVAL
+
+
+def test_null_context_is_refused_without_touching_a_device(lib):
+    """Every call that takes a context refuses a null one with JF_EINVAL (host check, no CUDA call)."""
+    from paper_2512_14681_gb300 import _lib as J
+
+    one = (C.c_int32 * 4)(1, 2, 3, 4)
+    out = (C.c_int32 * 4)()
+    f = (C.c_float * 4)()
+    n = C.c_int()
+    d = C.c_double()
+    ll = C.c_longlong()
+    blk = J.Block(0, 0, 1, -1)
+    gp = J.GenParams()
+    calls = {
+        "jf_init_random_weights": (None, 0, 0.02),
+        "jf_load_weights": (None, b"/nonexistent"),
+        "jf_save_weights": (None, b"/nonexistent"),
+        "jf_get_weights": (None, 0, 0, 1, f),
+        "jf_prefill": (None, 0, one, 4, out),
+        "jf_truncate": (None, 0, 0),
+        "jf_seq_len": (None, 0, C.byref(n)),
+        "jf_jacobi_step": (None, 0, 1, C.byref(blk), one, out, out, out, None, None),
+        "jf_forward_logits": (None, 0, 1, one, None, None, out),
+        "jf_generate": (None, 1, None, one, C.byref(gp), out, None),
+        "jf_generate_device": (None, 1, None, one, C.byref(gp), None, None),
+        "jf_set_profiling": (None, 1),
+        "jf_kernel_time": (None, 0, C.byref(d), C.byref(ll)),
+    }
+    for name, args in calls.items():
+        assert getattr(lib, name)(*args) == J.JF_EINVAL, name
+    assert lib.jf_last_error(None) == b"null context"
+    lib.jf_destroy(None)

@@ -454,17 +454,14 @@ __global__ void __launch_bounds__(128) k_attn_f32(const AttnParams a, int n_rows
     const int kp = kb + lane;
     float s = -INFINITY;
     const float* kr = nullptr;
-    const float* vr = nullptr;
     if (kp <= pos) {
       if (kp < ch.pos0) {
         const int page = a.page_table[(size_t)ch.seq * a.pages_per_seq + (kp >> 4)];
         const size_t off = (((size_t)page * a.Hkv + kvh) * kPage + (kp & 15)) * hd;
         kr = Kp + off;
-        vr = Vp + off;
       } else {
         const size_t off = ((size_t)(ch.row0 + kp - ch.pos0) * a.Hkv + kvh) * hd;
         kr = Ki + off;
-        vr = Vi + off;
       }
       float dot = 0.f;
       for (int i = 0; i < hd; ++i) dot = fmaf(q[i], kr[i], dot);
@@ -495,7 +492,6 @@ __global__ void __launch_bounds__(128) k_attn_f32(const AttnParams a, int n_rows
       if (lane + 32 < hd) o1 = fmaf(pj, vrow[lane + 32], o1);
     }
     m = mn;
-    (void)vr;
   }
   float* out = reinterpret_cast<float*>(a.out) + ((size_t)r * a.Hq + h) * hd;
   const float il = l > 0.f ? 1.f / l : 0.f;

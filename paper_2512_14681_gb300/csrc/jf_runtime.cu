@@ -44,7 +44,6 @@ enum ProfClass : int {
   PC_NORM = 8, PC_OTHER = 9, kProfClasses = 10
 };
 constexpr int kMaxStateInts = 32768;
-constexpr int kRandomTidMax = 8 + 16 * 4096;
 
 size_t rup(size_t x, size_t a) { return (x + a - 1) / a * a; }
 int cdiv(long long a, long long b) { return (int)((a + b - 1) / b); }

@@ -251,18 +251,19 @@ def test_attention_block_with_zero_queries_is_causal_mean():
 
 
 def test_mlp_block_closed_form():
-    """One layer, attention output zero, W_gate = W_up = W_down = I: x + silu(h) * h."""
+    """One layer, attention output zero, W_gate = I, W_up = 2 I, W_down = 3 I: x + 3 silu(h) (2 h).
+    The gate and up scales differ, so SiLU applied to the wrong branch is caught."""
     cfg = O.ModelConfig(n_layers=1, d_model=6, n_heads=2, n_kv_heads=2, head_dim=2, d_ff=6, vocab=16)
     m = O.Model(cfg).init_random(4, 0.5)
     r, k = m.shape(O.layer_tid(0, O.L_WO))
     m.set_tensor(O.layer_tid(0, O.L_WO), np.zeros(r * k))
-    for w in (O.L_WG, O.L_WU, O.L_WD):
-        m.set_tensor(O.layer_tid(0, w), np.eye(6))
+    for w, sc in ((O.L_WG, 1.0), (O.L_WU, 2.0), (O.L_WD, 3.0)):
+        m.set_tensor(O.layer_tid(0, w), sc * np.eye(6))
     toks = np.array([1, 9, 4], dtype=np.int32)
     out = O.forward(m, O.Cache(m, 8, 8), toks, np.arange(3), want_hidden=True)
     x = m.get_tensor(O.T_EMBED).reshape(16, 6)[toks]
     h = x / np.sqrt(np.mean(x * x, axis=1, keepdims=True) + cfg.rms_eps)
-    assert np.allclose(out.hidden, x + h / (1 + np.exp(-h)) * h, atol=1e-13)
+    assert np.allclose(out.hidden, x + 3.0 * (h / (1 + np.exp(-h))) * (2.0 * h), atol=1e-13)
 
 
 def test_positions_enter_through_relative_rotation():
@@ -307,3 +308,104 @@ def test_bf16_model_is_close_to_fp32_model():
     a = O.forward(m32, O.Cache(m32, 16, 8), toks, np.arange(8), want_logits=True)
     b = O.forward(m16, O.Cache(m16, 16, 8), toks, np.arange(8), want_logits=True)
     assert np.max(np.abs(a.logits - b.logits)) < 0.05
+
+
+def _bf(a):
+    """bf16 rounding (nearest, ties to even) by PyTorch, independent of the oracle's own routine."""
+    torch = pytest.importorskip("torch")
+    return torch.tensor(np.asarray(a, dtype=np.float64)).to(torch.bfloat16).to(torch.float64).numpy()
+
+
+def _bf16_layer_model(d, Hq, Hkv, hd, F, V):
+    cfg = O.ModelConfig(n_layers=1, d_model=d, n_heads=Hq, n_kv_heads=Hkv, head_dim=hd, d_ff=F, vocab=V, bf16=True)
+    return cfg, O.Model(cfg).init_random(6, 0.5)
+
+
+def test_bf16_final_norm_output_is_rounded():
+    """bf16 model, no layer contribution (W_o = W_down = 0), LM head = I: the logits are the final
+    RMSNorm output rounded to bf16, the precision the LM-head product takes its input in."""
+    cfg, m = _bf16_layer_model(8, 2, 2, 4, 8, 8)
+    for w in (O.L_WO, O.L_WD):
+        r, k = m.shape(O.layer_tid(0, w))
+        m.set_tensor(O.layer_tid(0, w), np.zeros(r * k))
+    m.set_tensor(O.T_LMHEAD, np.eye(8))
+    toks = np.array([1, 5, 2], dtype=np.int32)
+    out = O.forward(m, O.Cache(m, 8, 8), toks, np.arange(3), want_logits=True)
+    x = m.get_tensor(O.T_EMBED).reshape(8, 8)[toks]
+    h = np.stack([r * (1.0 / math.sqrt(float(np.dot(r, r)) / 8 + cfg.rms_eps)) for r in x])
+    assert np.max(np.abs(h - _bf(h))) > 1e-4              # the rounding is visible in this case
+    assert np.allclose(out.logits, _bf(h), rtol=0, atol=1e-12)
+
+
+def test_bf16_rounding_points_of_the_attention_block():
+    """bf16 model, d = hd = 2, one head, two tokens; W_q = I, W_k = [[0.75, 0], [0, 0]], W_v = 0.75 I,
+    W_o = I, MLP zero. Token 1 = (0, 1) has key 0 exactly, so row 1's softmax over keys {0, 1} has
+    the closed form p0 = e^s / (e^s + 1), s = q1 . k0 / sqrt(2). q, k and v are rounded to bf16
+    after the rotary embedding, and so is the attention output."""
+    cfg, m = _bf16_layer_model(2, 1, 1, 2, 2, 4)
+    A, B = np.array([1.0625, 0.3125]), np.array([0.0, 1.0])
+    E = np.zeros((4, 2))
+    E[0], E[1], E[2], E[3] = A, B, [0.5, 0.25], [-1.0, 2.0]
+    m.set_tensor(O.T_EMBED, E.ravel())
+    m.set_tensor(O.layer_tid(0, O.L_WQ), np.eye(2).ravel())
+    m.set_tensor(O.layer_tid(0, O.L_WK), np.array([0.75, 0.0, 0.0, 0.0]))
+    m.set_tensor(O.layer_tid(0, O.L_WV), (0.75 * np.eye(2)).ravel())
+    m.set_tensor(O.layer_tid(0, O.L_WO), np.eye(2).ravel())
+    for w in (O.L_WG, O.L_WU, O.L_WD):
+        m.set_tensor(O.layer_tid(0, w), np.zeros(4))
+    out = O.forward(m, O.Cache(m, 8, 8), np.array([0, 1], dtype=np.int32), np.arange(2), want_hidden=True)
+
+    def norm(x):
+        return _bf(x * (1.0 / math.sqrt(float(np.dot(x, x)) / 2 + cfg.rms_eps)))
+
+    h0, h1 = norm(A), norm(B)
+    c, sn = math.cos(1.0), math.sin(1.0)                      # position 1, frequency theta^0 = 1
+    q1 = _bf(np.array([h1[0] * c - h1[1] * sn, h1[1] * c + h1[0] * sn]))
+    k0 = _bf(np.array([0.75 * h0[0], 0.0]))                   # position 0: no rotation
+    assert abs(k0[0] - 0.75 * h0[0]) > 1e-4                    # the key needs rounding in this case
+    v0, v1 = _bf(0.75 * h0), _bf(0.75 * h1)
+    s = (q1[0] * k0[0] + q1[1] * k0[1]) * (1.0 / math.sqrt(2.0))
+    mx = max(s, 0.0)
+    p0, p1 = math.exp(s - mx), math.exp(0.0 - mx)
+    att1 = _bf((p0 * v0 + p1 * v1) / (p0 + p1))
+    assert np.max(np.abs(att1 - (p0 * v0 + p1 * v1) / (p0 + p1))) > 1e-4
+    assert np.allclose(out.hidden[0], A + v0, rtol=0, atol=1e-12)   # row 0 sees only itself
+    assert np.allclose(out.hidden[1], B + att1, rtol=0, atol=1e-12)
+
+
+def test_bf16_swiglu_product_is_rounded():
+    """bf16 model, attention output zero, W_gate = I, W_up = 2 I, W_down = 3 I: the hidden state is
+    x + 3 bf16(silu(h) 2h) with h the bf16 RMSNorm output."""
+    cfg, m = _bf16_layer_model(6, 2, 2, 2, 6, 16)
+    r, k = m.shape(O.layer_tid(0, O.L_WO))
+    m.set_tensor(O.layer_tid(0, O.L_WO), np.zeros(r * k))
+    for w, sc in ((O.L_WG, 1.0), (O.L_WU, 2.0), (O.L_WD, 3.0)):
+        m.set_tensor(O.layer_tid(0, w), sc * np.eye(6))
+    toks = np.array([1, 9, 4], dtype=np.int32)
+    out = O.forward(m, O.Cache(m, 8, 8), toks, np.arange(3), want_hidden=True)
+    x = m.get_tensor(O.T_EMBED).reshape(16, 6)[toks]
+    h = _bf(np.stack([r * (1.0 / math.sqrt(float(np.dot(r, r)) / 6 + cfg.rms_eps)) for r in x]))
+    silu = np.vectorize(lambda t: t / (1.0 + math.exp(-t)))
+    prod = silu(h) * (2.0 * h)
+    assert np.max(np.abs(prod - _bf(prod))) > 1e-4
+    assert np.allclose(out.hidden, x + 3.0 * _bf(prod), rtol=0, atol=1e-12)
+
+
+def test_bf16_kv_cache_holds_bf16_values():
+    """The KV cache of a bf16 model is bf16 (the precision the kernels store pages in): every committed
+    K (after the rotary embedding) and V value equals its own bf16 rounding, while the same entries of
+    the fp32 model do not all do so."""
+    for bf16 in (True, False):
+        cfg = O.ModelConfig(n_layers=2, d_model=64, n_heads=4, n_kv_heads=2, head_dim=16, d_ff=96, vocab=64,
+                            bf16=bf16)
+        m = O.Model(cfg).init_random(9, 0.3)
+        c = O.Cache(m, 16, 16)
+        toks = I.prompt_tokens(cfg.vocab, 7, seed=5)
+        O.forward(m, c, toks, np.arange(7))
+        c.commit(np.arange(7, dtype=np.int32))
+        vals = np.concatenate([c.entry(l, w, p).ravel() for l in range(2) for w in (0, 1) for p in range(7)])
+        assert np.count_nonzero(vals) > 0.9 * vals.size
+        if bf16:
+            assert np.array_equal(vals, _bf(vals))
+        else:
+            assert not np.array_equal(vals, _bf(vals))

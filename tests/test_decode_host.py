@@ -97,8 +97,12 @@ def run_device(hd, pr, prompts, truths, stationary, V, script=None, wrong=wrong_
         for s, _, nr, _ in chains:
             rows[s] += nr
         cur_tok = [int(t) for t in tok[:M]]
-        pred = np.array(chain_predictions(cur_tok, [int(x) for x in pos[:M]], chains, committed, truths, stationary,
-                                          wrong), dtype=np.int32)
+        cur_pos = [int(x) for x in pos[:M]]
+        pred = np.array(chain_predictions(cur_tok, cur_pos, chains, committed, truths, stationary, wrong),
+                        dtype=np.int32)
+        fwd = [[] for _ in range(ns)]  # per sequence: its chains' (tokens, positions) in order
+        for s_, r0, nr, _ in chains:
+            fwd[s_].append((cur_tok[r0:r0 + nr], cur_pos[r0:r0 + nr]))
         prev_out = nout.copy()
         hd.hd_accept(_p(pred), M)
         view()
@@ -111,7 +115,7 @@ def run_device(hd, pr, prompts, truths, stationary, V, script=None, wrong=wrong_
             assert p_at == len(committed[b]) and kk == k[b]
             committed[b] += cur_tok[row0:row0 + kk]  # the rows the KV commit copies into the cache
             recs[b].append(dict(M=rows[b], k=int(k[b]), winner=int(win[b]),
-                                out=[int(t) for t in out[b, prev_out[b]:nout[b]]]))
+                                out=[int(t) for t in out[b, prev_out[b]:nout[b]]], fwd=fwd[b]))
             done[b] = bool(nout[b] >= pr.max_new or (pr.eos_id >= 0 and pr.eos_id in out[b, :nout[b]]))
     else:
         raise AssertionError("decoding did not terminate")
@@ -119,13 +123,40 @@ def run_device(hd, pr, prompts, truths, stationary, V, script=None, wrong=wrong_
     return recs, [[int(t) for t in out[b, :nout[b]]] for b in range(ns)]
 
 
-def run_oracle(pr, prompt, truth_seq, stationary, V, monkeypatch, wrong=wrong_const):
+def run_oracle(pr, prompt, truth_seq, stationary, V, monkeypatch, wrong=wrong_const, calls=None):
     toy = toy_module(truth_seq, stationary, wrong)
     toy.sm64 = J.O.sm64  # the injection rule's generator stays the oracle's own
+    if calls is not None:
+        inner = toy.forward
+
+        def forward(model, cache, tokens, pos, seg=None, anc=None, **kw):
+            calls.append(([int(t) for t in tokens], [int(x) for x in pos],
+                          [0] * len(tokens) if seg is None else [int(v) for v in seg]))
+            return inner(model, cache, tokens, pos, seg, anc, **kw)
+
+        toy.forward = forward
     monkeypatch.setattr(J, "O", toy)
     model = types.SimpleNamespace(cfg=types.SimpleNamespace(vocab=V))
     truth = truth_seq[len(prompt):] if pr.init == "inject" else None
     return J.JacobiDecoder(model, prompt, pr, truth=truth).run()
+
+
+def _segments(tokens, pos, seg):
+    """The oracle's rows of one forward as the kernels' chains: the real-active block with its pseudo
+    blocks (segments 0 .. n_main-1, consecutive positions), then one chain per candidate."""
+    n_main = 0
+    while n_main < len(seg) and (n_main == 0 or seg[n_main] >= seg[n_main - 1]) and \
+            (n_main == 0 or pos[n_main] == pos[n_main - 1] + 1):
+        n_main += 1
+    out = [(tokens[:n_main], pos[:n_main])]
+    i = n_main
+    while i < len(seg):
+        j = i
+        while j < len(seg) and seg[j] == seg[i]:
+            j += 1
+        out.append((tokens[i:j], pos[i:j]))
+        i = j
+    return out
 
 
 @pytest.mark.parametrize("path", CASES, ids=[os.path.basename(c)[:-4] for c in CASES])
@@ -193,11 +224,14 @@ def test_device_state_machine_equals_oracle_loop(hd, case_seed, monkeypatch):
 
     recs, toks = run_device(hd, pr, prompts, truths, stationary, V, wrong=wrong)
     for b in range(ns):
-        want = run_oracle(pr, prompts[b], truths[b], stationary[b], V, monkeypatch, wrong)
+        calls = []
+        want = run_oracle(pr, prompts[b], truths[b], stationary[b], V, monkeypatch, wrong, calls)
         assert toks[b] == want.tokens, f"sequence {b}: {pr}"
         assert len(recs[b]) == len(want.iters), f"sequence {b}: {pr}"
+        fwds = calls[1:]  # the first call is the prefill
         for i, (have, it) in enumerate(zip(recs[b], want.iters)):
             assert (have["M"], have["k"], have["winner"]) == (it.M, it.k, it.winner), f"seq {b} iteration {i}: {pr}"
+            assert have["fwd"] == _segments(*fwds[i]), f"seq {b} iteration {i}: rows of the forward differ: {pr}"
 
 
 def test_step_mode_verification(hd):

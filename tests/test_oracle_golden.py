@@ -63,7 +63,8 @@ def test_golden_traces_are_lossless():
         spec = parse(path)
         assert spec["tokens"] == spec["truth"][: len(spec["tokens"])], path
         flat = [t for it in spec["iters"] for t in it["committed"]]
-        assert flat == spec["tokens"], path
+        assert flat == spec["truth"][: len(flat)], path            # every committed token is the truth
+        assert flat[: len(spec["tokens"])] == spec["tokens"], path  # the output stops inside the last commit
 
 
 # Plausible mistakes in the decoding loop, each planted (in memory, on the CPU) into a copy of the

@@ -192,6 +192,18 @@ jf_status jf_generate_device(jf_ctx* ctx, int n_seqs, const int32_t* d_prompts, 
 jf_status jf_set_profiling(jf_ctx* ctx, int enable);
 jf_status jf_kernel_time(jf_ctx* ctx, int kernel_class, double* total_ms, long long* launches);
 
+/* Timeline of the forward's kernels, for libraries built with JF_TIMELINE defined (the default
+ * build returns JF_EUNSUPPORTED and records nothing). records: device memory for
+ * JF_TL_MAX_RECORDS records of 40 bytes {uint32 kernel id, block, SM, pad; uint64 entry time,
+ * time past the dependency wait, exit time (ns, %globaltimer)}, written by thread 0 of every CTA;
+ * counter: a device int32 the caller zeroes, incremented once per record (records past the
+ * maximum are dropped). Kernel ids: 1 RMSNorm, 2 RMSNorm adding split-K partials, 3 QKV finish,
+ * 5 attention, 10 + e projection GEMM with epilogue e (13 SwiGLU, 14 argmax, 15 split-K partials),
+ * 20 embedding, 21 acceptance, 22 KV commit. (NULL, NULL) stops recording. Not tied to a context:
+ * the setting is process-wide and reaches CUDA graphs captured before it. */
+#define JF_TL_MAX_RECORDS 2000000
+jf_status jf_tl_enable(void* records, void* counter);
+
 #ifdef __cplusplus
 }
 #endif

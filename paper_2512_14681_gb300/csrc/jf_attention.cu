@@ -206,6 +206,7 @@ __global__ void __maxnreg__(200) k_attn_tc(const AttnParams a) {
   __shared__ float red_max[2][kAttnQRows];
   __shared__ float red_l[2][kAttnQRows];
 
+  JF_TL_ENTRY();
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int j = (int)cluster_rank();
   const int ui = (int)cluster_id_x();
@@ -245,6 +246,7 @@ __global__ void __maxnreg__(200) k_attn_tc(const AttnParams a) {
     cp_async_commit();
   }
   pdl_wait();  // queries and in-flight keys come from the QKV projection
+  JF_TL_WAITED();
   if (n_steps > 0) {
     const bf16* Q = reinterpret_cast<const bf16*>(a.q);
     for (int i = tid; i < kAttnQRows * 16; i += ATT_THREADS) {
@@ -425,6 +427,7 @@ __global__ void __maxnreg__(200) k_attn_tc(const AttnParams a) {
   }
   tc_fence_after();
   if (warp == 0) tmem_dealloc(tmem, TC_TMEM_COLS);
+  JF_TL_EXIT(TL_ATTN);
 }
 
 // fp32 path: one warp per (row, query head); keys in absolute order, 32 at a time.
@@ -500,6 +503,10 @@ __global__ void __launch_bounds__(128) k_attn_f32(const AttnParams a, int n_rows
 }
 
 }  // namespace
+
+#ifdef JF_TIMELINE
+JF_TL_SETTER(tl_set_attn)
+#endif
 
 cudaError_t launch_attn_tc(const AttnParams& a, int units_bound, cudaStream_t st) {
   cudaLaunchConfig_t cfg = {};

@@ -184,7 +184,9 @@ __global__ void k_gen_accept(const GenCfg g, int* state, const int* gpred, int M
   int* S = sm;
   int* gp = sm + g.state_stride;  // predictions of the current forward
   __shared__ int s_nch, s_rows;
+  JF_TL_ENTRY();
   pdl_wait();
+  JF_TL_WAITED();
   const SeqLayout L = seq_layout(g.n, g.K, g.C, g.G, g.pool_size);
   for (int i = threadIdx.x; i < M_cur; i += blockDim.x) gp[i] = gpred[i];
   if (threadIdx.x == 0) s_nch = 0;
@@ -357,6 +359,7 @@ __global__ void k_gen_accept(const GenCfg g, int* state, const int* gpred, int M
     res->all_done = all_done;
     res->err = *err;
   }
+  JF_TL_EXIT(TL_ACCEPT);
   pdl_launch_dependents();
 }
 
@@ -396,7 +399,9 @@ __global__ void k_step_accept(const StepBlocks* sbp, const int* tok, const int* 
 __global__ void k_commit(const CommitInfo* commit, const uint8_t* k_inf, const uint8_t* v_inf, uint8_t* k_pages,
                          uint8_t* v_pages, const int* page_table, int pages_per_seq, int n_pages, int max_rows, int Hkv,
                          int hd, int es, int* seq_len, int* err) {
+  JF_TL_ENTRY();
   pdl_wait();
+  JF_TL_WAITED();
   const int l = blockIdx.x, b = blockIdx.y;
   const CommitInfo ci = commit[b];
   const size_t head_bytes = (size_t)hd * es;
@@ -420,6 +425,7 @@ __global__ void k_commit(const CommitInfo* commit, const uint8_t* k_inf, const u
     *reinterpret_cast<uint4*>(v_pages + dst) = *reinterpret_cast<const uint4*>(vsrc + src);
   }
   if (l == 0 && threadIdx.x == 0) seq_len[b] = ci.P + ci.k;
+  JF_TL_EXIT(TL_COMMIT);
   pdl_launch_dependents();
 }
 
@@ -437,6 +443,10 @@ cudaLaunchConfig_t pdl_cfg(dim3 grid, dim3 block, size_t smem, cudaStream_t st, 
 }
 
 }  // namespace
+
+#ifdef JF_TIMELINE
+JF_TL_SETTER(tl_set_decode)
+#endif
 
 cudaError_t launch_gen_init(const GenCfg& g, int* state, const int* q0, const int* seq_len, const int* prompt_last,
                             int* tok, int* pos, Chain* chains, int* n_chains_dev, IterResult* res, int* err,

@@ -22,6 +22,56 @@ JF_DEV uint64_t jf_globaltimer() {
   return t;
 }
 
+// Kernel ids of the timeline records.
+enum TlKernel : unsigned {
+  TL_NORM = 1, TL_NORM_ACC = 2, TL_QKV_FINISH = 3, TL_ATTN = 5, TL_GEMM = 10 /* + epilogue kind */,
+  TL_EMBED = 20, TL_ACCEPT = 21, TL_COMMIT = 22
+};
+
+// Timeline of the forward's kernels, compiled in only with -DJF_TIMELINE (the default build has
+// none of it): thread 0 of every CTA records its kernel id, block, SM, entry time, the time it got
+// past its dependency wait and its exit time, into a caller buffer set by jf_tl_enable().
+#ifdef JF_TIMELINE
+struct TlRec {
+  unsigned kid, blk, smid, pad;
+  unsigned long long t0, t1, t2;
+};
+constexpr int kTlMaxRecords = 2000000;
+static __device__ TlRec* jf_tl_buf;  // one pair per translation unit, set by its own setter
+static __device__ int* jf_tl_idx;
+JF_DEV void jf_tl_record(unsigned kid, uint64_t t0, uint64_t t1) {
+  if (!jf_tl_buf) return;
+  const uint64_t t2 = jf_globaltimer();
+  unsigned sm;
+  asm volatile("mov.u32 %0, %%smid;" : "=r"(sm));
+  const int i = atomicAdd(jf_tl_idx, 1);
+  if (i < kTlMaxRecords) jf_tl_buf[i] = TlRec{kid, blockIdx.x, sm, 0u, t0, t1, t2};
+}
+#define JF_TL_ENTRY()                       \
+  const uint64_t jf_tl_t0 = jf_globaltimer(); \
+  uint64_t jf_tl_t1 = 0
+#define JF_TL_WAITED() (jf_tl_t1 = jf_globaltimer())
+#define JF_TL_EXIT(kid)                                               \
+  do {                                                                \
+    if (threadIdx.x == 0) jf_tl_record((unsigned)(kid), jf_tl_t0, jf_tl_t1); \
+  } while (0)
+#define JF_TL_SETTER(name)                                                     \
+  cudaError_t name(void* records, void* counter) {                             \
+    cudaError_t e = cudaMemcpyToSymbol(jf_tl_buf, &records, sizeof(void*));   \
+    return e != cudaSuccess ? e : cudaMemcpyToSymbol(jf_tl_idx, &counter, sizeof(void*)); \
+  }
+#else
+#define JF_TL_ENTRY() \
+  do {                \
+  } while (0)
+#define JF_TL_WAITED() \
+  do {                 \
+  } while (0)
+#define JF_TL_EXIT(kid) \
+  do {                  \
+  } while (0)
+#endif
+
 // ------------------------------------------------------------------------------------------
 // Programmatic dependent launch. Every kernel of the chain calls pdl_wait() before it reads
 // anything an earlier kernel wrote (and before it exits), so completion stays transitive.

@@ -66,8 +66,10 @@ __global__ void k_rope_table(float2* tab, int n_pos, int half, double theta) {
 template <typename T>
 __global__ void k_embed(const T* __restrict__ E, const int* __restrict__ tok, float* __restrict__ x, int d, int V,
                         int* err) {
+  JF_TL_ENTRY();
   pdl_launch_dependents();
   pdl_wait();
+  JF_TL_WAITED();
   const int r = blockIdx.x;
   int t = tok[r];
   if (t < 0 || t >= V) {
@@ -77,6 +79,7 @@ __global__ void k_embed(const T* __restrict__ E, const int* __restrict__ tok, fl
   const T* src = E + (size_t)t * d;
   float* dst = x + (size_t)r * d;
   for (int i = threadIdx.x; i < d; i += blockDim.x) dst[i] = act_to_f32(src[i]);
+  JF_TL_EXIT(TL_EMBED);
 }
 
 // y[r, :] = x[r, :] / sqrt(mean(x[r, :]^2) + eps) * gain, rounded to the activation type.
@@ -136,8 +139,10 @@ __global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(float* __restrict__ x,
                                                           T* __restrict__ y, int d, float eps, SplitPartials sp,
                                                           int row0) {
   __shared__ float red[NORM_THREADS / 32];
+  JF_TL_ENTRY();
   pdl_launch_dependents();  // the next projection may launch now and prefetch its weights
   pdl_wait();
+  JF_TL_WAITED();
   const int r = row0 + blockIdx.x;
   const int nv = d >> 2;
   float4* xr = reinterpret_cast<float4*>(x + (size_t)r * d);
@@ -200,6 +205,7 @@ __global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(float* __restrict__ x,
       store4(yr + 4 * i, make_float4(v[j].x * rs * g.x, v[j].y * rs * g.y, v[j].z * rs * g.z, v[j].w * rs * g.w));
     }
   }
+  JF_TL_EXIT(KS > 0 ? TL_NORM_ACC : TL_NORM);
 }
 
 // Finish of the QKV projection from its split-K partials (EPI_PARTIAL, head_dim 128 = one weight
@@ -212,8 +218,10 @@ __global__ void __launch_bounds__(128) k_qkv_finish(SplitPartials sp, const int*
                                                      const float2* __restrict__ rope, bf16* __restrict__ q,
                                                      bf16* __restrict__ k, bf16* __restrict__ v, int M, int Hq,
                                                      int Hkv) {
+  JF_TL_ENTRY();
   pdl_launch_dependents();
   pdl_wait();
+  JF_TL_WAITED();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int slots = Hq + 2 * Hkv;
   const int job = blockIdx.x * 4 + warp;
@@ -254,6 +262,7 @@ __global__ void __launch_bounds__(128) k_qkv_finish(SplitPartials sp, const int*
     dst = v + ((size_t)m * Hkv + (hs - Hq - Hkv)) * 128;
   }
   store4(dst + lane * 4, a);
+  JF_TL_EXIT(TL_QKV_FINISH);
 }
 
 template <typename K, typename... Args>
@@ -271,6 +280,10 @@ cudaError_t launch_pdl(K kernel, dim3 grid, dim3 block, cudaStream_t st, Args...
 }
 
 }  // namespace
+
+#ifdef JF_TIMELINE
+JF_TL_SETTER(tl_set_elem)
+#endif
 
 cudaError_t launch_init_weights(void* dst, bool is_bf16, long long rows, long long cols, uint64_t seed, uint64_t tid,
                                 double stdv, long long grp, long long grp_stride, long long grp_off, cudaStream_t st) {

@@ -399,6 +399,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + S);
   const uint32_t tfull0 = smem_u32(bars + 2 * S), tempty0 = smem_u32(bars + 2 * S + 2);
   const int total_units = p.n_tiles * p.m_tiles * p.k_splits;
+  JF_TL_ENTRY();
   // The next kernel may launch as soon as every CTA of this grid is resident: its CTAs take the
   // SMs this grid leaves, prefetch their own weights and park in their dependency wait, so no
   // launch latency is paid after the last tile (it writes nothing before that wait).
@@ -525,6 +526,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   } else {
     // epilogue warps 0-3
     pdl_wait();
+    JF_TL_WAITED();
     if constexpr (EPI == EPI_ARGMAX) {
       argmax_init_slots(p.epi, 0, p.M, blockIdx.x, gridDim.x, tid, 128);
       epi_sync();
@@ -550,6 +552,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   tc_fence_before();
   __syncthreads();
   if (warp == 4) tmem_dealloc(tmem, Cfg::TMEM_COLS);
+  JF_TL_EXIT(TL_GEMM + EPI);
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -651,6 +654,10 @@ cudaError_t prep_tc() {
 }
 
 }  // namespace
+
+#ifdef JF_TIMELINE
+JF_TL_SETTER(tl_set_gemm)
+#endif
 
 // Opt the tcgen05 kernels into their dynamic shared-memory sizes (once per process, outside any
 // stream capture).

@@ -118,6 +118,13 @@ cudaError_t launch_gemm_bf16(const CUtensorMap& tmA, const CUtensorMap& tmB, con
                              cudaStream_t st);
 cudaError_t launch_gemm_f32(const float* W, const float* X, const GemmParams& p, cudaStream_t st);
 int gemm_bn_for(int M);
+#ifdef JF_TIMELINE
+// Timeline builds: point each translation unit's record buffer / counter at caller memory.
+cudaError_t tl_set_gemm(void* records, void* counter);
+cudaError_t tl_set_attn(void* records, void* counter);
+cudaError_t tl_set_elem(void* records, void* counter);
+cudaError_t tl_set_decode(void* records, void* counter);
+#endif
 size_t gemm_smem_bytes(int bn);
 int gemm_default_splits(int n_tiles, int kb_total);
 bool encode_tmap_bf16(CUtensorMap* tm, const void* ptr, long long K, long long rows, int box_rows);

@@ -1355,6 +1355,20 @@ jf_status jf_set_profiling(jf_ctx* c, int enable) {
   return JF_OK;
 }
 
+jf_status jf_tl_enable(void* records, void* counter) {
+#ifdef JF_TIMELINE
+  if ((records == nullptr) != (counter == nullptr)) return JF_EINVAL;
+  if (jf::tl_set_gemm(records, counter) != cudaSuccess || jf::tl_set_attn(records, counter) != cudaSuccess ||
+      jf::tl_set_elem(records, counter) != cudaSuccess || jf::tl_set_decode(records, counter) != cudaSuccess)
+    return JF_ECUDA;
+  return JF_OK;
+#else
+  (void)records;
+  (void)counter;
+  return JF_EUNSUPPORTED;
+#endif
+}
+
 jf_status jf_kernel_time(jf_ctx* c, int cls, double* total_ms, long long* launches) {
   if (!c || cls < 0 || cls >= kProfClasses || !total_ms || !launches) return fail(c, JF_EINVAL, "bad arguments");
   *total_ms = c->prof_ms[cls];

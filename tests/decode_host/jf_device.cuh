@@ -25,6 +25,17 @@ int scripted_inject(const jf::GenCfg& g, int seq, int x, int P0, int it, int* er
 #define gridDim jf_host::grid_dim
 
 inline void __syncthreads() {}
+// the kernels' optional timeline records are not part of this build
+enum TlKernel : unsigned { TL_ACCEPT = 21, TL_COMMIT = 22 };
+#define JF_TL_ENTRY() \
+  do {                \
+  } while (0)
+#define JF_TL_WAITED() \
+  do {                 \
+  } while (0)
+#define JF_TL_EXIT(kid) \
+  do {                  \
+  } while (0)
 inline void pdl_wait() {}
 inline void pdl_launch_dependents() {}
 inline void jf_set_error(int* err, int code) {

@@ -131,7 +131,8 @@ def run_oracle(pr, prompt, truth_seq, stationary, V, monkeypatch, wrong=wrong_co
 
         def forward(model, cache, tokens, pos, seg=None, anc=None, **kw):
             calls.append(([int(t) for t in tokens], [int(x) for x in pos],
-                          [0] * len(tokens) if seg is None else [int(v) for v in seg]))
+                          [0] * len(tokens) if seg is None else [int(v) for v in seg],
+                          None if anc is None else [int(v) for v in anc]))
             return inner(model, cache, tokens, pos, seg, anc, **kw)
 
         toy.forward = forward
@@ -139,6 +140,25 @@ def run_oracle(pr, prompt, truth_seq, stationary, V, monkeypatch, wrong=wrong_co
     model = types.SimpleNamespace(cfg=types.SimpleNamespace(vocab=V))
     truth = truth_seq[len(prompt):] if pr.init == "inject" else None
     return J.JacobiDecoder(model, prompt, pr, truth=truth).run()
+
+
+def _tree_equals_chains(tokens, pos, seg, anc):
+    """The paper's tree mask (a row sees its own segment causally and every ancestor segment) and the
+    kernels' chain rule (a row sees the rows of its chain at positions up to its own) give the same
+    visible in-flight rows for this forward."""
+    M = len(tokens)
+    anc = anc or [0] * (max(seg) + 1)
+    chains = _segments(tokens, pos, seg)
+    chain_of, start = [], 0
+    for ci, (t, _) in enumerate(chains):
+        chain_of += [ci] * len(t)
+    for i in range(M):
+        for j in range(M):
+            tree = (seg[j] == seg[i] and pos[j] <= pos[i]) or (seg[j] != seg[i] and (anc[seg[i]] >> seg[j]) & 1)
+            chain = chain_of[j] == chain_of[i] and pos[j] <= pos[i]
+            if bool(tree) != chain:
+                return False
+    return True
 
 
 def _segments(tokens, pos, seg):
@@ -239,7 +259,8 @@ def test_device_state_machine_equals_oracle_loop(hd, case_seed, monkeypatch):
         fwds = calls[1:]  # the first call is the prefill
         for i, (have, it) in enumerate(zip(recs[b], want.iters)):
             assert (have["M"], have["k"], have["winner"]) == (it.M, it.k, it.winner), f"seq {b} iteration {i}: {pr}"
-            assert have["fwd"] == _segments(*fwds[i]), f"seq {b} iteration {i}: rows of the forward differ: {pr}"
+            assert have["fwd"] == _segments(*fwds[i][:3]), f"seq {b} iteration {i}: rows of the forward differ: {pr}"
+            assert _tree_equals_chains(*fwds[i]), f"seq {b} iteration {i}: tree mask != chains: {pr}"
 
 
 def test_step_mode_verification(hd):

@@ -675,7 +675,10 @@ jf_status get_graph(jf_ctx* c, const GenCfg& g, int M, int n_seqs, GraphRec** ou
   }
   e = cudaGraphInstantiate(&rec.exec, graph, 0);
   cudaGraphDestroy(graph);
-  if (e != cudaSuccess) return fail(c, JF_ECUDA, std::string("graph instantiate: ") + cudaGetErrorString(e));
+  if (e != cudaSuccess) {
+    for (cudaEvent_t ev : rec.ev) cudaEventDestroy(ev);
+    return fail(c, JF_ECUDA, std::string("graph instantiate: ") + cudaGetErrorString(e));
+  }
   auto ins = c->graphs.emplace(key, rec);
   *out = &ins.first->second;
   return JF_OK;

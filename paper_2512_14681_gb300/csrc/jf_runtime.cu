@@ -904,6 +904,13 @@ jf_status jf_create(const jf_model_config* model, const jf_runtime_config* rt, j
     if (cudaStreamCreateWithFlags(&c->st, cudaStreamNonBlocking) != cudaSuccess) { delete c; return JF_ECUDA; }
     c->own_stream = true;
   }
+  // a failure from here on releases what the context already holds
+  auto abandon = [c](jf_status s) {
+    if (c->res_host) cudaFreeHost(c->res_host);
+    if (c->own_stream) cudaStreamDestroy(c->st);
+    delete c;
+    return s;
+  };
   c->w_embed = at<void>(c, O.w_embed);
   c->w_lm = at<void>(c, O.w_lm);
   c->g_final = at<float>(c, O.g_final);
@@ -919,10 +926,10 @@ jf_status jf_create(const jf_model_config* model, const jf_runtime_config* rt, j
     if (D.bf16) {
       bool ok = make_tmap(&w.tm_qkv, w.qkv, D.d, D.nqkv, kTileN) && make_tmap(&w.tm_o, w.o, D.nq, D.d, kTileN) &&
                 make_tmap(&w.tm_gu, w.gu, D.d, 2 * D.F, kTileN) && make_tmap(&w.tm_dn, w.dn, D.F, D.d, kTileN);
-      if (!ok) { delete c; return JF_ECUDA; }
+      if (!ok) return abandon(JF_ECUDA);
     }
   }
-  if (D.bf16 && !make_tmap(&c->tm_lm, c->w_lm, D.d, D.V, kTileN)) { delete c; return JF_ECUDA; }
+  if (D.bf16 && !make_tmap(&c->tm_lm, c->w_lm, D.d, D.V, kTileN)) return abandon(JF_ECUDA);
   c->rope = at<float2>(c, O.rope);
   c->k_pages = at<void>(c, O.k_pages);
   c->v_pages = at<void>(c, O.v_pages);
@@ -961,7 +968,10 @@ jf_status jf_create(const jf_model_config* model, const jf_runtime_config* rt, j
   c->sb_dev = at<StepBlocks>(c, O.step_blocks);
   c->sres_dev = at<StepResult>(c, O.step_res);
   c->committed_dev = at<int>(c, O.committed);
-  if (cudaMallocHost(&c->res_host, sizeof(IterResult)) != cudaSuccess) { delete c; return JF_ENOMEM; }
+  if (cudaMallocHost(&c->res_host, sizeof(IterResult)) != cudaSuccess) {
+    c->res_host = nullptr;
+    return abandon(JF_ENOMEM);
+  }
   init_pages(c);
   // zero the small control buffers; fill the page table with -1
   cudaError_t e = cudaSuccess;
@@ -983,12 +993,7 @@ jf_status jf_create(const jf_model_config* model, const jf_runtime_config* rt, j
   if (e == cudaSuccess) e = gemm_prepare();
   if (e == cudaSuccess) e = attn_prepare();
   if (e == cudaSuccess) e = cudaStreamSynchronize(c->st);
-  if (e != cudaSuccess) {
-    cudaFreeHost(c->res_host);
-    if (c->own_stream) cudaStreamDestroy(c->st);
-    delete c;
-    return JF_ECUDA;
-  }
+  if (e != cudaSuccess) return abandon(JF_ECUDA);
   *out = c;
   return JF_OK;
 }

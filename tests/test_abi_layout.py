@@ -41,3 +41,23 @@ def test_ctypes_structs_match_the_header(tmp_path):
         assert got[(cname, "sizeof")] == J.C.sizeof(py), cname
         for f, _ in py._fields_:
             assert got[(cname, f)] == getattr(py, f).offset, (cname, f)
+
+
+@pytest.mark.skipif(shutil.which("gcc") is None, reason="needs gcc")
+def test_oracle_config_struct_matches_its_c_definition(tmp_path):
+    from oracle import oracle as O
+
+    fields = [f for f, _ in O._Cfg._fields_]
+    lines = ['#include <stddef.h>', '#include <stdio.h>', '#include "%s"' % os.path.join(ROOT, "oracle", "jf_oracle.c"),
+             "int main(void) {", '  printf("sizeof %zu\\n", sizeof(orc_config));']
+    lines += [f'  printf("{f} %zu\\n", offsetof(orc_config, {f}));' for f in fields]
+    lines += ["  return 0;", "}"]
+    src = tmp_path / "orc_layout.c"
+    src.write_text("\n".join(lines) + "\n")
+    exe = tmp_path / "orc_layout"
+    subprocess.run(["gcc", "-std=c11", str(src), "-o", str(exe), "-lm"], check=True, capture_output=True)
+    got = dict(ln.split() for ln in subprocess.run([str(exe)], check=True, capture_output=True,
+                                                   text=True).stdout.split("\n") if ln.strip())
+    assert int(got["sizeof"]) == O.C.sizeof(O._Cfg)
+    for f in fields:
+        assert int(got[f]) == getattr(O._Cfg, f).offset, f

@@ -1,0 +1,53 @@
+"""The GPU parity tests' comparison rule (tests/parity.py), on synthetic generations (no GPU):
+tokens equal up to the first divergence, which must sit at one of the oracle's near-ties; committed
+counts equal for every iteration that ends before it."""
+import types
+
+import pytest
+
+from tests.parity import compare_generation, flag_tol
+
+
+def ref(tokens, counts, margins):
+    return types.SimpleNamespace(tokens=list(tokens), counts=list(counts), margins=list(margins))
+
+
+def test_identical_generation_passes():
+    r = ref([5, 6, 7, 8, 9], [2, 2, 1], [1.0] * 5)
+    assert compare_generation([5, 6, 7, 8, 9], [2, 2, 1], r, bf16=True) is None
+
+
+def test_divergence_at_a_near_tie_is_flagged_and_later_counts_are_free():
+    tol = flag_tol(True)
+    r = ref([5, 6, 7, 8, 9, 10], [2, 3, 1], [1.0, 1.0, 1.0, 1.0, tol / 2, 1.0])
+    rep = []
+    # token 4 differs at a near-tie; iteration 1 (tokens 2..4) may then commit a different count
+    assert compare_generation([5, 6, 7, 8, 3, 3], [2, 1, 9], r, bf16=True, report=rep) == 4
+    assert rep == [("flagged", 4, tol / 2)]
+
+
+def test_divergence_at_a_clear_decision_fails():
+    r = ref([5, 6, 7, 8], [2, 2], [1.0, 1.0, 1.0, 1.0])
+    with pytest.raises(AssertionError):
+        compare_generation([5, 6, 0, 8], [2, 2], r, bf16=False)
+
+
+def test_fp32_tolerance_is_tighter_than_bf16():
+    r = ref([5, 6, 7], [3], [1.0, 1e-3, 1.0])
+    assert compare_generation([5, 0, 7], [3], r, bf16=True) == 1        # 1e-3 < 2 * 3e-2
+    with pytest.raises(AssertionError):
+        compare_generation([5, 0, 7], [3], r, bf16=False)              # 1e-3 > 2 * 1e-4
+
+
+def test_count_mismatch_before_the_divergence_fails():
+    r = ref([5, 6, 7, 8, 9], [1, 2, 2], [1.0, 1.0, 1.0, 1.0, 1e-9])
+    with pytest.raises(AssertionError):
+        compare_generation([5, 6, 7, 8, 0], [2, 1, 2], r, bf16=True)   # iteration 0 ends before token 4
+
+
+def test_length_and_count_mismatch_without_divergence_fail():
+    r = ref([5, 6, 7], [2, 1], [1.0] * 3)
+    with pytest.raises(AssertionError):
+        compare_generation([5, 6], [2, 1], r, bf16=True)
+    with pytest.raises(AssertionError):
+        compare_generation([5, 6, 7], [1, 2], r, bf16=True)

@@ -1057,24 +1057,27 @@ std::vector<int> all_tids(const Dims& D) {
 
 long long dev_row(const TensorLoc& t, long long r) { return (r / t.grp) * t.grp_stride + (r % t.grp) + t.grp_off; }
 
-// Whole tensor between its device rows and a dense host buffer [rows][cols]: one strided 2-D copy
-// of the full groups of t.grp rows, one more for a partial last group.
-cudaError_t copy_tensor(const TensorLoc& t, int es, void* host, cudaMemcpyKind kind) {
+// Whole tensor between its device rows and a dense host buffer [rows][cols], ordered on stream st
+// (the caller synchronises it before using or releasing the host buffer): one strided 2-D copy of
+// the full groups of t.grp rows, one more for a partial last group.
+cudaError_t copy_tensor(const TensorLoc& t, int es, void* host, cudaMemcpyKind kind, cudaStream_t st) {
   const size_t rb = (size_t)t.cols * es;
   const bool to_dev = kind == cudaMemcpyHostToDevice;
   if (t.grp >= t.rows) {
     char* dev = t.base + (size_t)t.grp_off * rb;
-    return to_dev ? cudaMemcpy(dev, host, (size_t)t.rows * rb, kind) : cudaMemcpy(host, dev, (size_t)t.rows * rb, kind);
+    return to_dev ? cudaMemcpyAsync(dev, host, (size_t)t.rows * rb, kind, st)
+                  : cudaMemcpyAsync(host, dev, (size_t)t.rows * rb, kind, st);
   }
   const long long full = t.rows / t.grp, tail = t.rows % t.grp;
   const size_t gw = (size_t)t.grp * rb, dp = (size_t)t.grp_stride * rb;
   char* h = reinterpret_cast<char*>(host);
   char* dev = t.base + (size_t)t.grp_off * rb;
-  cudaError_t e = to_dev ? cudaMemcpy2D(dev, dp, h, gw, gw, (size_t)full, kind) : cudaMemcpy2D(h, gw, dev, dp, gw, (size_t)full, kind);
+  cudaError_t e = to_dev ? cudaMemcpy2DAsync(dev, dp, h, gw, gw, (size_t)full, kind, st)
+                         : cudaMemcpy2DAsync(h, gw, dev, dp, gw, (size_t)full, kind, st);
   if (e != cudaSuccess || tail == 0) return e;
   char* dt = t.base + (size_t)dev_row(t, full * t.grp) * rb;
   char* ht = h + (size_t)full * gw;
-  return to_dev ? cudaMemcpy(dt, ht, (size_t)tail * rb, kind) : cudaMemcpy(ht, dt, (size_t)tail * rb, kind);
+  return to_dev ? cudaMemcpyAsync(dt, ht, (size_t)tail * rb, kind, st) : cudaMemcpyAsync(ht, dt, (size_t)tail * rb, kind, st);
 }
 
 struct FileHeader {
@@ -1153,7 +1156,8 @@ jf_status jf_save_weights(jf_ctx* c, const char* path) {
     tensor_loc(c, tid, &t);
     const int es = t.gain ? 4 : c->D.es;
     buf.resize((size_t)t.rows * t.cols * es);
-    if (copy_tensor(t, es, buf.data(), cudaMemcpyDeviceToHost) != cudaSuccess) {
+    if (copy_tensor(t, es, buf.data(), cudaMemcpyDeviceToHost, c->st) != cudaSuccess ||
+        cudaStreamSynchronize(c->st) != cudaSuccess) {
       std::fclose(f);
       return fail(c, JF_ECUDA, "copy of weights failed");
     }
@@ -1197,8 +1201,9 @@ jf_status jf_load_weights(jf_ctx* c, const char* path) {
   for (size_t i = 0; i < locs.size(); ++i) {
     const TensorLoc& t = locs[i];
     const int es = t.gain ? 4 : c->D.es;
-    CK(copy_tensor(t, es, data[i].data(), cudaMemcpyHostToDevice));
+    CK(copy_tensor(t, es, data[i].data(), cudaMemcpyHostToDevice, c->st));
   }
+  CK(cudaStreamSynchronize(c->st));  // the host buffers are released on return
   c->weights_ready = true;
   return JF_OK;
 }

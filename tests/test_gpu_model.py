@@ -169,3 +169,46 @@ def test_invalid_step_is_rejected_without_state_change(pair):
             ctx.jacobi_step(0, blocks, np.array(draft, dtype=np.int32))
         assert ctx.seq_len(0) == 10
     ctx.truncate(0, 0)
+
+
+def test_weight_file_roundtrip_and_refused_files(pair, tmp_path):
+    """jf_save_weights / jf_load_weights: the saved file loads back bit for bit over other weights; a
+    truncated file and a file of another shape are refused with JF_EIO and leave the weights as they
+    were (the whole file is read and checked before any upload)."""
+    from paper_2512_14681_gb300 import _lib as J
+
+    shape, ctx, model = pair
+    tids = [0, 1, 2] + [8 + w for w in range(9)]  # every tensor kind of layer 0
+
+    def snap():
+        out = {}
+        for t in tids:
+            n = model.get_tensor(t).size
+            head = min(n, 4096)
+            out[t] = np.concatenate([ctx.get_weights(t, 0, head), ctx.get_weights(t, n - head, head)])
+        return out
+
+    path = str(tmp_path / "w.jfw")
+    ctx.save_weights(path)
+    before = snap()
+    ctx.init_random_weights(I.WEIGHT_SEED + 7, I.WEIGHT_STD)
+    other = snap()
+    assert any(not np.array_equal(before[t], other[t]) for t in tids if t != 2)
+    ctx.load_weights(path)
+    for t in tids:
+        assert np.array_equal(snap()[t], before[t]), t
+    data = open(path, "rb").read()
+    bad = str(tmp_path / "bad.jfw")
+    open(bad, "wb").write(data[: len(data) // 2])
+    with pytest.raises(J.JfError) as ei:
+        ctx.load_weights(bad)
+    assert ei.value.status == J.JF_EIO
+    wrong = bytearray(data)
+    wrong[4 * 4: 4 * 4 + 4] = (int.from_bytes(data[16:20], "little") + 64).to_bytes(4, "little")  # d_model
+    open(bad, "wb").write(bytes(wrong))
+    with pytest.raises(J.JfError) as ei:
+        ctx.load_weights(bad)
+    assert ei.value.status == J.JF_EIO
+    after = snap()
+    for t in tids:
+        assert np.array_equal(after[t], before[t]), t

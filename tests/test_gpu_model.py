@@ -212,3 +212,25 @@ def test_weight_file_roundtrip_and_refused_files(pair, tmp_path):
     after = snap()
     for t in tids:
         assert np.array_equal(after[t], before[t]), t
+
+
+def test_refused_prefill_and_truncate_leave_the_sequence(pair):
+    """Host checks before any launch: a prompt past max_ctx (JF_ECAPACITY), an out-of-range token
+    (JF_EINVAL), a truncate past the committed length and a bad sequence slot (JF_EINVAL)."""
+    from paper_2512_14681_gb300 import _lib as J
+
+    shape, ctx, model = pair
+    ctx.truncate(0, 0) if ctx.seq_len(0) else None
+    ctx.prefill(0, I.prompt_tokens(shape.vocab, 12, seed=31))
+    cases = [
+        (J.JF_ECAPACITY, lambda: ctx.prefill(0, I.prompt_tokens(shape.vocab, 512, seed=32))),  # 12 + 512 > 512
+        (J.JF_EINVAL, lambda: ctx.prefill(0, np.array([1, shape.vocab], dtype=np.int32))),
+        (J.JF_EINVAL, lambda: ctx.truncate(0, 13)),
+        (J.JF_EINVAL, lambda: ctx.prefill(5, np.array([1, 2], dtype=np.int32))),               # max_seqs = 2
+    ]
+    for status, call in cases:
+        with pytest.raises(J.JfError) as ei:
+            call()
+        assert ei.value.status == status
+        assert ctx.seq_len(0) == 12
+    ctx.truncate(0, 0)

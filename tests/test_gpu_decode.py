@@ -32,6 +32,12 @@ MODES = {
     # the shape of the paper's inference configuration (K = 2, r = 0.85, 4 verified n-grams), small n
     "inj_mr_k2_r085_c4": dict(block_size=8, n_blocks=2, spawn_ratio=0.85, pool_size=16, cand_per_iter=4,
                               init="inject", inject_p=0.3, seed=5),
+    # recycling in the running window, and n-grams shorter than the block
+    "window_rr": dict(block_size=6, mode="window", pool_size=8, cand_per_iter=1),
+    "inj_window_rr_g5": dict(block_size=8, mode="window", pool_size=16, cand_per_iter=2, ngram_len=5,
+                             init="inject", inject_p=0.3, seed=6),
+    "inj_mb3_r05_rr_g3": dict(block_size=8, n_blocks=3, spawn_ratio=0.5, pool_size=8, cand_per_iter=2, ngram_len=3,
+                              init="inject", inject_p=0.3, seed=7),
 }
 
 

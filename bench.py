@@ -318,6 +318,8 @@ def run_gpu(args, rank, world, local_rank):
     # per-iteration roofline: every weight byte + the committed KV read once per iteration
     n_iter = first.iterations
     it_ms = first.decode_ms / max(n_iter, 1)
+    # per-iteration device time of each graph replay (CUDA events around it) in the logged step
+    it_rep = first.iter_ms if first.iter_ms is not None and len(first.iter_ms) else np.array([it_ms])
     kv_tok = shape.kv_bytes_per_token()
     p_avg = PROMPT_LEN + NEW / 2.0   # committed length averaged over the generation
     it_bytes = shape.weight_bytes() + kv_tok * p_avg
@@ -340,6 +342,7 @@ def run_gpu(args, rank, world, local_rank):
                 "d2h_bytes_per_step": int(NEW * 4)},
         "gpu_launches": int(launches),
         "iteration": {"count_per_step": n_iter, "tokens_per_iteration": NEW / max(n_iter, 1), "ms": it_ms,
+                      "replay_p50_ms": float(np.median(it_rep)), "replay_p90_ms": float(np.percentile(it_rep, 90)),
                       "prefill_ms": first.prefill_ms, "bytes": it_bytes, "achieved_gbs": it_gbs,
                       "frac_of_" + peak_kind: it_gbs / peak, "frac_of_8tbs": it_gbs / NOMINAL_HBM_GBS},
         "roofline": {"bound": "hbm", "kernel": "gate/up projection GEMM (tcgen05, SwiGLU epilogue)",

@@ -158,9 +158,10 @@ typedef struct {
 
 /* Statistics of one generation. accepted (optional caller buffer [accepted_cap][n_seqs]):
  * tokens committed per iteration (-1 once a sequence is done); rows (optional [accepted_cap]):
- * in-flight rows of each iteration. Times from CUDA events on the context's stream.
- * kernel_launches: libjf kernels launched by the call (prefill, setup and every node of every
- * replayed decode-iteration graph). */
+ * in-flight rows of each iteration; iter_ms (optional [accepted_cap]): device time of each
+ * iteration's graph replay, from CUDA events recorded around it. Times from CUDA events on the
+ * context's stream. kernel_launches: libjf kernels launched by the call (prefill, setup and every
+ * node of every replayed decode-iteration graph). */
 typedef struct {
   int iterations;
   int32_t* accepted;
@@ -168,6 +169,7 @@ typedef struct {
   int accepted_cap;
   double prefill_ms, decode_ms;
   long long kernel_launches;
+  float* iter_ms;
 } jf_gen_stats;
 
 /* Prefill then Jacobi-decode n_seqs independent sequences (slots 0 .. n_seqs-1, which are reset)

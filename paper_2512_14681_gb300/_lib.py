@@ -62,7 +62,7 @@ class GenParams(C.Structure):
 class GenStats(C.Structure):
     _fields_ = [("iterations", C.c_int), ("accepted", C.POINTER(C.c_int32)), ("rows", C.POINTER(C.c_int32)),
                 ("accepted_cap", C.c_int), ("prefill_ms", C.c_double), ("decode_ms", C.c_double),
-                ("kernel_launches", C.c_longlong)]
+                ("kernel_launches", C.c_longlong), ("iter_ms", C.POINTER(C.c_float))]
 
 
 _lib = None

@@ -703,7 +703,7 @@ void accumulate_profile(jf_ctx* c, GraphRec* g) {
 // Timing events of one call; destroyed on every return path (an event still pending in the stream
 // is released once the device reaches it).
 struct CallEvents {
-  cudaEvent_t e[3] = {nullptr, nullptr, nullptr};
+  cudaEvent_t e[5] = {nullptr, nullptr, nullptr, nullptr, nullptr};
   ~CallEvents() {
     for (cudaEvent_t x : e)
       if (x) cudaEventDestroy(x);
@@ -776,6 +776,11 @@ jf_status generate_impl(jf_ctx* c, int n_seqs, const int32_t* const* h_prompts, 
   CK(cudaEventCreate(&ev.e[1]));
   CK(cudaEventCreate(&ev.e[2]));
   const cudaEvent_t e0 = ev.e[0], e1 = ev.e[1], e2 = ev.e[2];
+  const bool time_iters = stats && stats->iter_ms && stats->accepted_cap > 0;
+  if (time_iters) {  // around each graph replay, outside the graph
+    CK(cudaEventCreate(&ev.e[3]));
+    CK(cudaEventCreate(&ev.e[4]));
+  }
   CK(cudaEventRecord(e0, c->st));
   std::vector<int> q0(n_seqs), plast(n_seqs);
   long long off = 0;
@@ -827,9 +832,16 @@ jf_status generate_impl(jf_ctx* c, int n_seqs, const int32_t* const* h_prompts, 
     if (M < 1 || M > D.R) return fail(c, JF_EDEVICE, "device produced an invalid row count");
     GraphRec* gr = nullptr;
     if ((s = get_graph(c, g, M, n_seqs, &gr)) != JF_OK) return s;
+    if (time_iters) CK(cudaEventRecord(ev.e[3], c->st));
     CK(cudaGraphLaunch(gr->exec, c->st));
+    if (time_iters) CK(cudaEventRecord(ev.e[4], c->st));
     c->launches += gr->kernels;
     CK(cudaStreamSynchronize(c->st));
+    if (time_iters && iters < stats->accepted_cap) {
+      float ms = 0.f;
+      CK(cudaEventElapsedTime(&ms, ev.e[3], ev.e[4]));
+      stats->iter_ms[iters] = ms;
+    }
     if (c->profiling) accumulate_profile(c, gr);
     rows_log.push_back(M);
     ++iters;

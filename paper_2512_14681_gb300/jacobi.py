@@ -25,6 +25,10 @@ def _i32p(a):
     return a.ctypes.data_as(C.POINTER(C.c_int32))
 
 
+def _f32p(a):
+    return a.ctypes.data_as(C.POINTER(C.c_float))
+
+
 @dataclass
 class Gen:
     """Generation parameters (see jf_gen_params in include/jf.h)."""
@@ -58,6 +62,7 @@ class GenOut:
     prefill_ms: float
     decode_ms: float
     kernel_launches: int = 0
+    iter_ms: np.ndarray | None = None  # [iterations] device time of each iteration's graph replay
 
 
 def model_config(shape: ModelShape) -> J.ModelConfig:
@@ -178,11 +183,12 @@ class Context:
         out = np.empty((n, gen.max_new), dtype=np.int32)
         acc = np.full((log_cap, n), -1, dtype=np.int32)
         rows = np.zeros(log_cap, dtype=np.int32)
-        st = J.GenStats(0, _i32p(acc), _i32p(rows), log_cap, 0.0, 0.0, 0)
+        ims = np.zeros(max(log_cap, 1), dtype=np.float32)
+        st = J.GenStats(0, _i32p(acc), _i32p(rows), log_cap, 0.0, 0.0, 0, _f32p(ims) if log_cap > 0 else None)
         self._c(self.lib.jf_generate(self.h, n, arr, _i32p(lens), C.byref(gp), _i32p(out), C.byref(st)))
         it = st.iterations
-        return GenOut(out, acc[: min(it, log_cap)], rows[: min(it, log_cap)], it, st.prefill_ms, st.decode_ms,
-                      st.kernel_launches)
+        k = min(it, log_cap)
+        return GenOut(out, acc[:k], rows[:k], it, st.prefill_ms, st.decode_ms, st.kernel_launches, ims[:k])
 
     def generate_device(self, d_prompts, prompt_lens, gen: Gen, d_out, d_truth=None, truth_len=0,
                         log_cap: int = 0):
@@ -192,12 +198,13 @@ class Context:
         n = lens.size
         acc = np.full((max(log_cap, 1), n), -1, dtype=np.int32)
         rows = np.zeros(max(log_cap, 1), dtype=np.int32)
-        st = J.GenStats(0, _i32p(acc), _i32p(rows), log_cap, 0.0, 0.0, 0)
+        ims = np.zeros(max(log_cap, 1), dtype=np.float32)
+        st = J.GenStats(0, _i32p(acc), _i32p(rows), log_cap, 0.0, 0.0, 0, _f32p(ims) if log_cap > 0 else None)
         self._c(self.lib.jf_generate_device(self.h, n, d_prompts.data_ptr(), _i32p(lens), C.byref(gp),
                                             d_out.data_ptr(), C.byref(st)))
         it = st.iterations
-        return GenOut(None, acc[: min(it, log_cap)], rows[: min(it, log_cap)], it, st.prefill_ms, st.decode_ms,
-                      st.kernel_launches)
+        k = min(it, log_cap)
+        return GenOut(None, acc[:k], rows[:k], it, st.prefill_ms, st.decode_ms, st.kernel_launches, ims[:k])
 
     def set_profiling(self, on: bool):
         self._c(self.lib.jf_set_profiling(self.h, 1 if on else 0))

@@ -71,6 +71,9 @@ def test_generate_matches_oracle(setup, mode):
     div = compare_generation(out.tokens[0], out.counts[:, 0], ref, shape.bf16, report)
     if div is None:
         assert out.rows.tolist() == [it.M for it in ref.iters]
+    # every iteration's graph replay was timed, and the replays fit inside the decode time
+    assert out.iter_ms.shape == (out.iterations,) and np.all(out.iter_ms > 0)
+    assert out.iter_ms.sum() <= out.decode_ms + 1e-3
     print(mode, "iterations", out.iterations, "flags", report)
 
 

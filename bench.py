@@ -384,14 +384,18 @@ def run_sweep(args):
     for P, n, B in SWEEP_POINTS:
         prompts = [I.prompt_tokens(shape.vocab, P, seed=100 + b) for b in range(B)]
         out = ctx.generate(prompts, Gen(block_size=n, mode="window", max_new=args.steps + args.warmup), log_cap=64)
-        it_ms = out.decode_ms / max(out.iterations, 1)
+        # median device time of the replays after the warm-up ones (the first iteration of a point also
+        # captures and instantiates its graph on the host, which the decode time would include)
+        reps = out.iter_ms[args.warmup:] if out.iter_ms is not None and len(out.iter_ms) > args.warmup else None
+        it_ms = float(np.median(reps)) if reps is not None else out.decode_ms / max(out.iterations, 1)
         kv = shape.kv_bytes_per_token() * (P + 2) * B
         by = shape.weight_bytes() + kv
         M = n * B
         flops = 2.0 * M * (shape.weight_bytes() / 2) + 4.0 * shape.head_dim * shape.n_heads * P * shape.n_layers * M
         t_bytes = by / (peak * 1e9) * 1e3
         t_flops = flops / 1.936e15 * 1e3
-        pts.append({"prompt": P, "block": n, "batch": B, "rows": M, "iteration_ms": it_ms, "bytes": by,
+        pts.append({"prompt": P, "block": n, "batch": B, "rows": M, "iteration_ms": it_ms,
+                    "iteration_ms_incl_host": out.decode_ms / max(out.iterations, 1), "bytes": by,
                     "gbs": by / (it_ms / 1000.0) / 1e9, "flops": flops,
                     "roofline_ms": max(t_bytes, t_flops), "bound": "hbm" if t_bytes >= t_flops else "tensor",
                     "frac_of_roofline": max(t_bytes, t_flops) / it_ms})

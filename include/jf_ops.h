@@ -45,8 +45,11 @@ jf_status jf_op_gemm(int dtype, const void* W, const void* X, float* Y, int N, i
  * loading libjf holds until the process exits; a shape whose jf_op_gemm_workspace_bytes() exceeds
  * it is refused with JF_ECAPACITY before any launch. The call allocates nothing (no cudaMalloc,
  * no cudaFree, no allocating library routine). Its first call on a device looks up the array's
- * device address (cudaGetSymbolAddress) and sets kernel attributes, so make that first call before
- * any stream capture. All calls share the array: calls that may overlap on the GPU (other streams,
+ * device address (cudaGetSymbolAddress) and sets that device's kernel attributes, so make that
+ * first call before any stream capture. Under CUDA's lazy module loading (the default) that first
+ * look-up may also be what loads libjf's device code onto the device and reserves the array there:
+ * make the first call at start-up, before another pool takes the device memory, or run with
+ * CUDA_MODULE_LOADING=EAGER so that the array is reserved when the library is loaded. All calls share the array: calls that may overlap on the GPU (other streams,
  * other threads) race on it and must be serialised by the caller; each call re-zeroes the tickets
  * it uses before its kernel runs. err_word and cuda_stream as in jf_op_gemm. */
 jf_status jf_op_gemm_noalloc(const void* W, const void* X, float* Y, int N, int K, int M, int k_splits,

@@ -14,6 +14,7 @@
 // by the weight shape alone, so a row's result does not depend on how many rows are in flight.
 #include "jf_device.cuh"
 #include "jf_internal.h"
+#include "jf_once.h"
 
 namespace jf {
 namespace {
@@ -659,9 +660,8 @@ cudaError_t prep_tc() {
 JF_TL_SETTER(tl_set_gemm)
 #endif
 
-// Opt the tcgen05 kernels into their dynamic shared-memory sizes (once per process, outside any
-// stream capture).
-cudaError_t gemm_prepare() {
+// Opt the tcgen05 kernels into their dynamic shared-memory sizes on the current device.
+static cudaError_t gemm_prepare_current() {
   cudaError_t e;
   if ((e = prep_tc<16>()) != cudaSuccess) return e;
   if ((e = prep_tc<32>()) != cudaSuccess) return e;
@@ -669,6 +669,17 @@ cudaError_t gemm_prepare() {
   if ((e = prep_tc<128>()) != cudaSuccess) return e;
   if ((e = prep_tc<160>()) != cudaSuccess) return e;
   return prep_tc<256>();
+}
+
+// The attributes are per device: set them once for each device the process uses (outside any
+// stream capture), whichever entry point reaches that device first.
+cudaError_t gemm_prepare() {
+  static PerDeviceOnce once;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const int r = once.run(dev, [] { return gemm_prepare_current(); });
+  return r < 0 ? cudaErrorInvalidDevice : static_cast<cudaError_t>(r);
 }
 
 int gemm_bn_for(int M) {

@@ -22,7 +22,6 @@ namespace {
 constexpr int kMaxDevices = 64;
 std::mutex g_mu;
 void* g_scratch_ptr[kMaxDevices] = {};
-bool g_prepared = false;
 
 size_t rup256(size_t x) { return (x + 255) / 256 * 256; }
 
@@ -36,10 +35,8 @@ jf_status scratch_for_current_device(void** out) {
     if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return JF_ECUDA;
     g_scratch_ptr[dev] = p;
   }
-  if (!g_prepared) {
-    if (gemm_prepare() != cudaSuccess) return JF_ECUDA;
-    g_prepared = true;
-  }
+  // kernel attributes are per device; gemm_prepare sets them once for each device it meets
+  if (gemm_prepare() != cudaSuccess) return JF_ECUDA;
   *out = g_scratch_ptr[dev];
   return JF_OK;
 }

@@ -1456,11 +1456,7 @@ jf_status jf_op_gemm(int dtype, const void* W, const void* X, float* Y, int N, i
   p.epi.ldy = N;
   cudaError_t e;
   if (dtype == JF_BF16) {
-    static bool prepared = false;
-    if (!prepared) {
-      if (gemm_prepare() != cudaSuccess) return JF_ECUDA;
-      prepared = true;
-    }
+    if (gemm_prepare() != cudaSuccess) return JF_ECUDA;  // once per device
     CUtensorMap tA, tB;
     if (!make_tmap(&tA, W, K, N, kTileN) || !make_tmap(&tB, X, K, M, bn)) return JF_ECUDA;
     e = launch_gemm_bf16(tA, tB, p, bn, st);

@@ -157,21 +157,25 @@ def aggregate_ranks(local_ms: float, local_tokens: int, dist=None, device=None):
 # ------------------------------------------------------------------------------------------
 # CPU oracle sample (the reference arm and the cpu_baseline object)
 # ------------------------------------------------------------------------------------------
-def oracle_sample(steps: int, warmup: int):
-    """Jacobi iterations of the oracle on the same 7B-shaped model and block size, with the
-    prompt cut to its first 16 tokens (the oracle cannot prefill 1024 tokens in minutes)."""
+def oracle_sample(steps: int, warmup: int, prompt_len: int = 16):
+    """Per-iteration figure of the oracle (fp64 C, OpenMP over the machine's host cores) on the headline
+    workload's model and decoding parameters: the 7B-shaped bf16 model, block n = 32, drafts injected
+    at p = 0.3 against the oracle's own greedy continuation. The oracle prefills the first
+    `prompt_len` prompt tokens (a 1,024-token prefill alone takes minutes on the host), runs `warmup`
+    untimed iterations, then times `steps` iterations. The seeds are fixed, so every run times the
+    same iterations with the same accepted counts."""
     from oracle import jacobi as OJ
     from oracle import oracle as O
     from paper_2512_14681_gb300 import inputs as I
 
     w = WORKLOADS[DEFAULT_WORKLOAD]
-    PROMPT_LEN, BLOCK, P_INJECT = w.prompt, w.block, w.p
+    BLOCK, P_INJECT = w.block, w.p
     shape = I.QWEN7B_BF16
     need = shape.weight_bytes() + (6 << 30)
     avail = os.sysconf("SC_AVPHYS_PAGES") * os.sysconf("SC_PAGE_SIZE")
     if avail < need:
         return None, f"host memory {avail >> 30} GiB < {need >> 30} GiB needed by the 7B oracle"
-    prompt = I.prompt_tokens(shape.vocab, PROMPT_LEN)[:16]
+    prompt = I.prompt_tokens(shape.vocab, w.prompt)[:prompt_len]
     model = O.Model(O.ModelConfig(**shape.oracle_kwargs())).init_random(I.WEIGHT_SEED, I.WEIGHT_STD)
     n_it = steps + warmup
     truth = OJ.generate_ar(model, prompt, n_it * BLOCK + 2 * BLOCK + 2).tokens
@@ -180,25 +184,48 @@ def oracle_sample(steps: int, warmup: int):
                            truth=truth)
     for _ in range(warmup):
         dec.step()
-    t0 = time.perf_counter()
-    toks = 0
+    times, toks = [], 0
     for _ in range(steps):
+        t0 = time.perf_counter()
         toks += dec.step().k
+        times.append(time.perf_counter() - t0)
+    dt = sum(times)
+    return dict(value=toks / dt, unit="tokens/s", cores=O.num_threads(), kind="oracle", dtype="f64",
+                ms_per_iteration=1000.0 * dt / steps, ms_per_iteration_median=1000.0 * statistics.median(times),
+                tokens_per_iteration=toks / steps, iterations=steps,
+                sample=f"{steps} timed Jacobi iterations after {warmup} untimed ones (n={BLOCK}, inject p={P_INJECT}, "
+                       f"seed {I.INJECT_SEED}) of the 7B-shaped model after a {prompt_len}-token prompt prefill; "
+                       f"{toks} tokens in {dt:.1f} s; fp64 arithmetic"), None
+
+
+def oracle_tiny_run():
+    """The oracle's full run of the tiny fp32 decoder (2 layers, d 256, vocabulary 4096; prompt of 32
+    tokens, block n = 8 with the repeated last prompt token as initial draft, 64 new tokens)."""
+    from oracle import jacobi as OJ
+    from oracle import oracle as O
+    from paper_2512_14681_gb300 import inputs as I
+
+    shape = I.TINY_F32
+    model = O.Model(O.ModelConfig(**shape.oracle_kwargs())).init_random(I.WEIGHT_SEED, I.WEIGHT_STD)
+    prompt = I.prompt_tokens(shape.vocab, 32, seed=I.PROMPT_SEED)
+    t0 = time.perf_counter()
+    res = OJ.generate_jacobi(model, prompt, OJ.GenParams(block_size=8, max_new=64))
     dt = time.perf_counter() - t0
-    return dict(value=toks / dt, unit="tokens/s", cores=O.num_threads(), kind="oracle",
-                sample=f"{steps} Jacobi iterations (n={BLOCK}, inject p={P_INJECT}) of the 7B-shaped model "
-                       f"after a 16-token prompt prefill; {toks} tokens in {dt:.1f} s"), None
+    return dict(value=len(res.tokens) / dt, unit="tokens/s", iterations=len(res.iters),
+                ms_per_iteration=1000.0 * dt / max(len(res.iters), 1), dtype="f64",
+                sample="tiny fp32 decoder, prompt 32, n=8, 64 new tokens, prefill included")
 
 
 def run_reference(args, rank):
     if rank != 0:
         return
-    res, why = oracle_sample(args.steps, args.warmup)
+    # one step = one Jacobi iteration of the oracle on the headline workload's model and parameters
+    res, why = oracle_sample(args.steps, args.warmup, args.cpu_baseline_prompt)
     if res is None:
         print(json.dumps({"impl": "reference", "unavailable": why}))
         return
     line = {"impl": "reference", "metric": METRIC, "value": res["value"], "unit": "tokens/s", "n_gpus": args.gpus,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 * 1.0 / max(res["value"], 1e-9),
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": res["ms_per_iteration"],
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "config": {"workload": DEFAULT_WORKLOAD, "sample": res["sample"]},
             "cpu_baseline": res, "e2e": {"value": res["value"], "unit": "tokens/s", "h2d_bytes_per_step": 0,
@@ -355,7 +382,9 @@ def run_gpu(args, rank, world, local_rank):
         "clocks": clocks,
     }
     if args.cpu_baseline and world == 1 and args.workload == DEFAULT_WORKLOAD and not args.layers:
-        cb, why = oracle_sample(args.cpu_baseline_iters, 0)
+        cb, why = oracle_sample(args.cpu_baseline_iters, 1, args.cpu_baseline_prompt)
+        if cb is not None:
+            cb["tiny_config"] = oracle_tiny_run()
         line["cpu_baseline"] = cb if cb is not None else {"unavailable": why}
     else:
         line["cpu_baseline"] = None
@@ -416,7 +445,10 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
-    ap.add_argument("--cpu-baseline-iters", type=int, default=2)
+    ap.add_argument("--cpu-baseline-iters", type=int, default=3)
+    ap.add_argument("--cpu-baseline-prompt", type=int, default=16,
+                    help="prompt tokens the oracle prefills before its timed iterations (1024 = the full prompt, "
+                         "several minutes on the host)")
     ap.add_argument("--layers", type=int, default=0, help="decoder layers (0 = the workload's; fewer = profiling case)")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD,
                     help="workload name or alias (" + ", ".join(ALIASES) + "); 'sweep' = fixed-shape latency sweep")

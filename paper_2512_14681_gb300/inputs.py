@@ -54,7 +54,11 @@ QWEN15B_BF16 = ModelShape("qwen2.5-1.5b-shape-bf16", 28, 1536, 12, 2, 128, 8960,
 # Qwen2.5-7B shape, bf16.
 QWEN7B_BF16 = ModelShape("qwen2.5-7b-shape-bf16", 28, 3584, 28, 4, 128, 18944, 152064, 1e-6, 1e6, True)
 
-SHAPES = {s.name: s for s in (TINY_F32, SMALL_BF16, QWEN15B_BF16, QWEN7B_BF16)}
+# Two layers of the Qwen2.5-7B shape (every per-layer width and the full vocabulary of the 7B model), so
+# that the oracle can check forwards at the 7B widths in seconds.
+QWEN7B_2L_BF16 = ModelShape("qwen2.5-7b-shape-2layer-bf16", 2, 3584, 28, 4, 128, 18944, 152064, 1e-6, 1e6, True)
+
+SHAPES = {s.name: s for s in (TINY_F32, SMALL_BF16, QWEN15B_BF16, QWEN7B_BF16, QWEN7B_2L_BF16)}
 
 WEIGHT_SEED = 0
 WEIGHT_STD = 0.02

@@ -48,3 +48,31 @@ def compare_generation(gpu_tokens, gpu_counts, ref, bf16: bool, report=None):
     if div is None:
         assert gc[: len(ref.counts)] == list(ref.counts)
     return div
+
+
+def compare_with_resync(run_gpu, run_oracle, prompt, max_new: int, bf16: bool, max_flags: int, report=None):
+    """Generation parity that continues past flagged near-ties.
+
+    run_oracle(prompt, max_new, offset) -> GenResult of the oracle's decoding loop;
+    run_gpu(prompt, max_new, offset) -> (tokens, per-iteration counts) of the device, both decoding
+    `max_new` tokens after `prompt` with the same parameters (`offset` = new tokens already decided
+    before `prompt` ends, for callers that index a truth continuation). Both runs are compared with
+    compare_generation. At a flagged divergence both sides are re-synchronised on the oracle's prefix
+    up to and including its decision at the near-tie (the device re-prefills that prefix), and the
+    comparison continues from there until max_new tokens are decided. At most `max_flags` flagged
+    positions are allowed; returns them as indexes into the new tokens."""
+    prompt = [int(t) for t in prompt]
+    done, flags = 0, []
+    while done < max_new:
+        ref = run_oracle(np.array(prompt, dtype=np.int32), max_new - done, done)
+        tokens, counts = run_gpu(np.array(prompt, dtype=np.int32), max_new - done, done)
+        div = compare_generation(tokens, counts, ref, bf16)
+        if div is None:
+            break
+        flags.append(done + div)
+        if report is not None:
+            report.append(("flagged", done + div, ref.margins[div]))
+        assert len(flags) <= max_flags, f"more than {max_flags} flagged near-ties: {flags}"
+        prompt += [int(t) for t in ref.tokens[: div + 1]]
+        done += div + 1
+    return flags

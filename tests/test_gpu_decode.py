@@ -1,7 +1,8 @@
 """jf_generate vs the oracle's decoding loops (Sec. 2.1 Eq. 3-4; Sec. 3.2 / Algorithm 1).
 
-Generated tokens and per-iteration accepted counts must be identical, except after a position
-where the oracle's top-1/top-2 logit margin is below twice the logit tolerance (flagged). Also
+Generated tokens and per-iteration accepted counts must be identical, except at a position where
+the oracle's top-1/top-2 logit margin is below twice the logit tolerance (flagged): there both
+sides are re-synchronised on the oracle's prefix and the comparison continues to the end. Also
 checked on the device alone: greedy Jacobi decoding in every mode reproduces the device's own
 greedy AR output token for token (the paper's fixed-point property), which holds exactly because
 each row's arithmetic is independent of the rows in flight with it.
@@ -12,7 +13,7 @@ import pytest
 from oracle import jacobi as OJ
 from oracle import oracle as O
 from paper_2512_14681_gb300 import inputs as I
-from tests.parity import compare_generation, need_gpu
+from tests.parity import compare_with_resync, need_gpu
 
 pytestmark = pytest.mark.gpu
 
@@ -62,19 +63,30 @@ def test_generate_matches_oracle(setup, mode):
     from paper_2512_14681_gb300.jacobi import Gen
 
     kw = dict(MODES[mode])
-    gen = Gen(max_new=48, **kw)
-    ogen = OJ.GenParams(max_new=48, **kw)
-    tr = truth.tokens if gen.init == "inject" else None
-    ref = OJ.generate_jacobi(model, prompt, ogen, truth=tr)
-    out = ctx.generate([prompt], gen, truth=None if tr is None else np.array([tr], dtype=np.int32))
-    report = []
-    div = compare_generation(out.tokens[0], out.counts[:, 0], ref, shape.bf16, report)
-    if div is None:
+    inject = kw.get("init") == "inject"
+    runs = []
+
+    def run_oracle(p, max_new, offset):
+        tr = truth.tokens[offset:] if inject else None
+        ref = OJ.generate_jacobi(model, p, OJ.GenParams(max_new=max_new, **kw), truth=tr)
+        runs.append(["oracle", ref])
+        return ref
+
+    def run_gpu(p, max_new, offset):
+        tr = np.array([truth.tokens[offset:]], dtype=np.int32) if inject else None
+        out = ctx.generate([p], Gen(max_new=max_new, **kw), truth=tr)
+        # every iteration's graph replay was timed, and the replays fit inside the decode time
+        assert out.iter_ms.shape == (out.iterations,) and np.all(out.iter_ms > 0)
+        assert out.iter_ms.sum() <= out.decode_ms + 1e-3
+        runs.append(["gpu", out])
+        return out.tokens[0], out.counts[:, 0]
+
+    # after a flagged near-tie both sides restart from the oracle's prefix; at most 2 such ties
+    flags = compare_with_resync(run_gpu, run_oracle, prompt, 48, shape.bf16, max_flags=2)
+    if not flags:
+        ref, out = runs[0][1], runs[1][1]
         assert out.rows.tolist() == [it.M for it in ref.iters]
-    # every iteration's graph replay was timed, and the replays fit inside the decode time
-    assert out.iter_ms.shape == (out.iterations,) and np.all(out.iter_ms > 0)
-    assert out.iter_ms.sum() <= out.decode_ms + 1e-3
-    print(mode, "iterations", out.iterations, "flags", report)
+    print(mode, "runs", len(runs) // 2, "flags", flags)
 
 
 def test_jacobi_equals_ar_on_device(setup):

@@ -51,3 +51,64 @@ def test_length_and_count_mismatch_without_divergence_fail():
         compare_generation([5, 6], [2, 1], r, bf16=True)
     with pytest.raises(AssertionError):
         compare_generation([5, 6, 7], [1, 2], r, bf16=True)
+
+
+# ---- re-synchronisation after flagged near-ties (compare_with_resync) ----------------------------
+from tests.parity import compare_with_resync  # noqa: E402
+
+
+def _runners(truth, margins, gpu_flip, count=2):
+    """Oracle: the truth continuation, `count` tokens per iteration. Device: the same, except that at
+    the absolute new-token indexes in gpu_flip it decides another token (and keeps its own branch)."""
+    calls = []
+
+    def oracle(prompt, max_new, offset):
+        toks = truth[offset: offset + max_new]
+        cnt = [count] * (len(toks) // count) + ([len(toks) % count] if len(toks) % count else [])
+        return ref(toks, cnt, margins[offset: offset + max_new])
+
+    def gpu(prompt, max_new, offset):
+        calls.append((len(prompt), max_new, offset))
+        toks = list(truth[offset: offset + max_new])
+        for i in gpu_flip:
+            if offset <= i < offset + max_new:
+                toks[i - offset:] = [t + 1000 for t in toks[i - offset:]]  # diverged branch
+                break
+        cnt = [count] * (len(toks) // count) + ([len(toks) % count] if len(toks) % count else [])
+        return toks, cnt
+
+    return oracle, gpu, calls
+
+
+def test_resync_continues_after_each_flagged_tie():
+    tol = flag_tol(True)
+    truth = list(range(10, 30))
+    margins = [1.0] * 20
+    margins[3] = margins[11] = tol / 4
+    oracle, gpu, calls = _runners(truth, margins, gpu_flip=[3, 11])
+    rep = []
+    flags = compare_with_resync(gpu, oracle, [1, 2, 3], 20, bf16=True, max_flags=2, report=rep)
+    assert flags == [3, 11]
+    # three runs: the whole generation, then from token 4 (prompt + 4 oracle tokens), then from 12
+    assert calls == [(3, 20, 0), (7, 16, 4), (15, 8, 12)]
+    assert [r[1] for r in rep] == [3, 11]
+
+
+def test_resync_still_fails_a_clear_divergence_after_a_tie():
+    tol = flag_tol(True)
+    truth = list(range(10, 30))
+    margins = [1.0] * 20
+    margins[3] = tol / 4
+    oracle, gpu, _ = _runners(truth, margins, gpu_flip=[3, 9])   # token 9 has a clear margin
+    with pytest.raises(AssertionError):
+        compare_with_resync(gpu, oracle, [1, 2, 3], 20, bf16=True, max_flags=4)
+
+
+def test_resync_bounds_the_number_of_flags():
+    tol = flag_tol(True)
+    truth = list(range(10, 30))
+    margins = [tol / 4] * 20
+    oracle, gpu, _ = _runners(truth, margins, gpu_flip=[2, 5, 8])
+    with pytest.raises(AssertionError):
+        compare_with_resync(gpu, oracle, [1], 20, bf16=True, max_flags=2)
+    assert compare_with_resync(gpu, oracle, [1], 20, bf16=True, max_flags=3) == [2, 5, 8]

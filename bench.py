@@ -393,7 +393,9 @@ def run_gpu(args, rank, world, local_rank):
         dist.destroy_process_group()
 
 
-SWEEP_POINTS = [(P, n, B) for P in (4096, 16384, 32768) for n in (32, 128) for B in (1, 4)]
+SWEEP_POINTS = [(P, n, B) for P in (4096, 8192, 16384, 32768) for n in (16, 32, 64, 128) for B in (1, 4)]
+# latency versus parallel tokens (the knee of App. D) at P = 4096, one sequence, n = rows
+KNEE_ROWS = [16, 32, 64, 128, 192, 256, 320, 384, 512]
 
 
 def run_sweep(args):
@@ -410,7 +412,8 @@ def run_sweep(args):
     ctx = Context(shape, max_seqs=4, max_ctx=maxP + 256, max_rows=512)
     ctx.init_random_weights(I.WEIGHT_SEED, I.WEIGHT_STD)
     pts = []
-    for P, n, B in SWEEP_POINTS:
+    points = [(P, n, B, "grid") for P, n, B in SWEEP_POINTS] + [(4096, r, 1, "knee") for r in KNEE_ROWS]
+    for P, n, B, kind in points:
         prompts = [I.prompt_tokens(shape.vocab, P, seed=100 + b) for b in range(B)]
         out = ctx.generate(prompts, Gen(block_size=n, mode="window", max_new=args.steps + args.warmup), log_cap=64)
         # median device time of the replays after the warm-up ones (the first iteration of a point also
@@ -423,15 +426,15 @@ def run_sweep(args):
         flops = 2.0 * M * (shape.weight_bytes() / 2) + 4.0 * shape.head_dim * shape.n_heads * P * shape.n_layers * M
         t_bytes = by / (peak * 1e9) * 1e3
         t_flops = flops / 1.936e15 * 1e3
-        pts.append({"prompt": P, "block": n, "batch": B, "rows": M, "iteration_ms": it_ms,
+        pts.append({"set": kind, "prompt": P, "block": n, "batch": B, "rows": M, "iteration_ms": it_ms,
                     "iteration_ms_incl_host": out.decode_ms / max(out.iterations, 1), "bytes": by,
                     "gbs": by / (it_ms / 1000.0) / 1e9, "flops": flops,
                     "roofline_ms": max(t_bytes, t_flops), "bound": "hbm" if t_bytes >= t_flops else "tensor",
                     "frac_of_roofline": max(t_bytes, t_flops) / it_ms})
         print(json.dumps(pts[-1]), file=sys.stderr, flush=True)
-    med = statistics.median(p["iteration_ms"] for p in pts)
+    med = statistics.median(p["iteration_ms"] for p in pts if p["set"] == "grid")
     print(json.dumps({"metric": "Jacobi-iteration latency sweep on the 7B shape (bf16, window mode)",
-                      "value": med, "unit": "ms (median over points)", "n_gpus": 1, "steps": args.steps,
+                      "value": med, "unit": "ms (median over the grid points)", "n_gpus": 1, "steps": args.steps,
                       "warmup": args.warmup, "higher_is_better": False, "dtype": "bf16", "data": "synthetic",
                       "config": {"workload": "qwen2.5-7b-shape-bf16 sweep P x n x B", "peak_gbs": peak,
                                  "peak_kind": peak_kind, "tensor_peak_tflops": 1936.4},

@@ -161,7 +161,18 @@ typedef struct {
  * in-flight rows of each iteration; iter_ms (optional [accepted_cap]): device time of each
  * iteration's graph replay, from CUDA events recorded around it. Times from CUDA events on the
  * context's stream. kernel_launches: libjf kernels launched by the call (prefill, setup and every
- * node of every replayed decode-iteration graph). */
+ * node of every replayed decode-iteration graph).
+ *
+ * Jacobi trajectories (Sec. 2.1: the points y^(0), y^(1), ... each block passes through until its
+ * fixed point; Sec. 3.1 trains on them). traj (optional, DEVICE int32 buffer lent for the call,
+ * traj_cap * (2 + 5 * traj_rows) elements): the device records iteration i < traj_cap at
+ * traj + i * (2 + 5 * traj_rows) as [M, i, seq[traj_rows], kind[traj_rows], pos[traj_rows],
+ * token[traj_rows], prediction[traj_rows]]: the M rows of that iteration's forward (M <= traj_rows;
+ * entries past M are left as they were) with the sequence slot, the kind (0 real-active draft,
+ * 1 pseudo-active block, 2 recycled candidate), absolute position, draft token and greedy
+ * prediction of each row. traj_rows must be >= n_seqs * (n_blocks * block_size +
+ * cand_per_iter * ngram_len) (JF_EINVAL otherwise). traj_iters (out): iterations recorded. Records
+ * are written by the acceptance kernel inside the iteration graph; no host copy is made. */
 typedef struct {
   int iterations;
   int32_t* accepted;
@@ -170,6 +181,9 @@ typedef struct {
   double prefill_ms, decode_ms;
   long long kernel_launches;
   float* iter_ms;
+  int32_t* traj;
+  int traj_cap, traj_rows;
+  int traj_iters;
 } jf_gen_stats;
 
 /* Prefill then Jacobi-decode n_seqs independent sequences (slots 0 .. n_seqs-1, which are reset)

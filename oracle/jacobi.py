@@ -69,6 +69,10 @@ class IterRecord:
     k_cand: list
     pseudo: list                 # pseudo-accepted counts per pseudo block
     committed: list
+    # the forward's rows, one entry per row: the Jacobi trajectory point y^(j) of the real-active block
+    # (Sec. 2.1), the pseudo blocks after it and the candidates, with their greedy predictions y^(j+1)
+    # (kind 0 = real-active, 1 = pseudo-active, 2 = recycled candidate)
+    rows: dict = field(default_factory=dict)
 
 
 @dataclass
@@ -340,7 +344,9 @@ class JacobiDecoder:
                 for i in order[:self.p.cand_per_iter]:
                     ent = self.pool[i]
                     self.cands.append(([self.q0] + ent[1:])[:Ln])
-        rec = IterRecord(len(tokens), k, winner, k_ra, k_c, pseudo_counts, committed)
+        kinds = [0] * len(ra.q) + [1] * (len(main_tok) - len(ra.q)) + [2] * (len(tokens) - len(main_tok))
+        rec = IterRecord(len(tokens), k, winner, k_ra, k_c, pseudo_counts, committed,
+                         dict(tokens=list(tokens), pos=list(pos), pred=g, kind=kinds, margin=mg))
         self.iters.append(rec)
         self.it = nit
         return rec

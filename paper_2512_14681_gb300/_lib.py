@@ -62,7 +62,8 @@ class GenParams(C.Structure):
 class GenStats(C.Structure):
     _fields_ = [("iterations", C.c_int), ("accepted", C.POINTER(C.c_int32)), ("rows", C.POINTER(C.c_int32)),
                 ("accepted_cap", C.c_int), ("prefill_ms", C.c_double), ("decode_ms", C.c_double),
-                ("kernel_launches", C.c_longlong), ("iter_ms", C.POINTER(C.c_float))]
+                ("kernel_launches", C.c_longlong), ("iter_ms", C.POINTER(C.c_float)), ("traj", C.c_void_p),
+                ("traj_cap", C.c_int), ("traj_rows", C.c_int), ("traj_iters", C.c_int)]
 
 
 _lib = None

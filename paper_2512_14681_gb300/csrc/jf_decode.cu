@@ -178,6 +178,60 @@ __global__ void k_gen_init(const GenCfg g, int* state, const int* q0, const int*
   }
 }
 
+// Jacobi trajectory record (Sec. 2.1: the points y^(0), y^(1), ... a block passes through, each with
+// the greedy predictions that give the next one): every row of the forward that just ran, with its
+// sequence, kind (0 real-active draft, 1 pseudo-active block, 2 recycled candidate), position, token
+// and prediction. Runs before the acceptance step rewrites the rows for the next forward.
+__device__ void record_trajectory(const GenCfg& g, const SeqLayout& L, const int* state, const int* gp, int M,
+                                  const int* tok, const int* pos) {
+  __shared__ int s_it;
+  if (threadIdx.x == 0) s_it = *g.traj_count;
+  __syncthreads();
+  const int it = s_it;
+  if (it < g.traj_cap) {
+    const int R = g.traj_rows;
+    const int Mr = M < R ? M : R;
+    int* rec = g.traj + (size_t)it * (2 + 5 * (size_t)R);
+    if (threadIdx.x == 0) {
+      rec[0] = M;
+      rec[1] = it;
+    }
+    for (int r = threadIdx.x; r < Mr; r += blockDim.x) {
+      rec[2 + r] = -1;
+      rec[2 + R + r] = -1;
+      rec[2 + 2 * R + r] = pos[r];
+      rec[2 + 3 * R + r] = tok[r];
+      rec[2 + 4 * R + r] = gp[r];
+    }
+    __syncthreads();
+    for (int b = 0; b < g.n_seqs; ++b) {
+      const int* S = state + (size_t)b * g.state_stride;
+      if (S[H_DONE]) continue;  // a finished sequence has no rows in this forward
+      const int mr0 = S[H_MAIN_ROW0], mlen = S[H_MAIN_LEN], lra = S[H_RA_LEN];
+      for (int r = threadIdx.x; r < mlen; r += blockDim.x) {
+        const int row = mr0 + r;
+        if (row >= 0 && row < Mr) {
+          rec[2 + row] = b;
+          rec[2 + R + row] = r < lra ? 0 : 1;
+        }
+      }
+      const int nc = S[H_NCAND];
+      for (int c = 0; c < nc; ++c) {
+        const int cr0 = S[L.cand_row0 + c], cl = S[L.cand_len + c];
+        for (int r = threadIdx.x; r < cl; r += blockDim.x) {
+          const int row = cr0 + r;
+          if (row >= 0 && row < Mr) {
+            rec[2 + row] = b;
+            rec[2 + R + row] = 2;
+          }
+        }
+      }
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) *g.traj_count = it + 1;
+}
+
 __global__ void k_gen_accept(const GenCfg g, int* state, const int* gpred, int M_cur, int* tok, int* pos,
                              Chain* chains, int* n_chains_dev, CommitInfo* commit, IterResult* res, int* err) {
   extern __shared__ int sm[];
@@ -191,6 +245,7 @@ __global__ void k_gen_accept(const GenCfg g, int* state, const int* gpred, int M
   for (int i = threadIdx.x; i < M_cur; i += blockDim.x) gp[i] = gpred[i];
   if (threadIdx.x == 0) s_nch = 0;
   __syncthreads();
+  if (g.traj) record_trajectory(g, L, state, gp, M_cur, tok, pos);
   const int n = g.n, G = g.G;
   int row_off = 0;
   int all_done = 1;

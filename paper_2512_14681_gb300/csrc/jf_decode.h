@@ -20,6 +20,12 @@ struct GenCfg {
   int* out_tokens;        // [n_seqs][max_new]
   int* iter_log;          // [max_iters][n_seqs] committed count (-1 = inactive)
   int max_iters;
+  // Trajectory record (optional, caller-lent device buffer): per iteration i < traj_cap, at
+  // traj + i * (2 + 5 * traj_rows): [M, i, seq[traj_rows], kind[traj_rows], pos[traj_rows],
+  // token[traj_rows], prediction[traj_rows]] for the M rows of that iteration's forward.
+  int* traj;
+  int traj_cap, traj_rows;
+  int* traj_count;        // device counter of recorded iterations (zeroed by the host per call)
 };
 
 // Layout of one sequence's state (ints). Header fields first.

@@ -110,7 +110,7 @@ struct Offsets {
   size_t k_inf, v_inf, x, h, q, att, act;
   size_t tok, pos, gpred, top2, chains, n_chains, attn_xchg;
   size_t gemm_ws, gemm_counter, am_v1, am_i1, am_v2, am_counter;
-  size_t logits, err;
+  size_t logits, err, traj_count;
   size_t gen_state, gen_out, gen_truth, gen_log, gen_q0, gen_plast, res, step_blocks, step_res, committed;
   size_t gemm_ws_bytes;
   size_t total;
@@ -221,6 +221,7 @@ Offsets plan_offsets(const Dims& D) {
   o.am_counter = p.take((size_t)max_mt * 4);
   o.logits = p.take((size_t)std::max(D.logits_rows, 1) * D.V * 4, 1024);
   o.err = p.take(16);
+  o.traj_count = p.take(16);
   o.gen_state = p.take((size_t)D.S * kMaxStateInts * 4);
   o.gen_out = p.take((size_t)D.S * D.max_ctx * 4);
   o.gen_truth = p.take((size_t)D.S * D.max_ctx * 4);
@@ -292,7 +293,7 @@ struct jf_ctx {
   int *am_i1, *am_counter;
   float* logits;
   int* err;
-  int *gen_state, *gen_out, *gen_truth, *gen_log, *gen_q0, *gen_plast;
+  int *gen_state, *gen_out, *gen_truth, *gen_log, *gen_q0, *gen_plast, *traj_count;
   IterResult* res_dev;
   StepBlocks* sb_dev;
   StepResult* sres_dev;
@@ -759,6 +760,9 @@ jf_status generate_impl(jf_ctx* c, int n_seqs, const int32_t* const* h_prompts, 
     jf_status s = check_tokens(c, p.truth, n_seqs * p.truth_len);
     if (s != JF_OK) return s;
   }
+  const bool want_traj = stats && stats->traj;
+  if (want_traj && (stats->traj_cap < 1 || stats->traj_rows < rows_per_seq * n_seqs))
+    return fail(c, JF_EINVAL, "trajectory buffer: traj_cap >= 1 and traj_rows >= the rows of one forward needed");
   // reset slots 0 .. n_seqs-1 and reserve their pages
   for (int b = 0; b < n_seqs; ++b) {
     release_pages(c, b, 0);
@@ -817,6 +821,13 @@ jf_status generate_impl(jf_ctx* c, int n_seqs, const int32_t* const* h_prompts, 
   g.max_rows = D.R; g.max_chains = D.max_chains; g.max_ctx = D.max_ctx;
   c->chains_bound = std::min(D.max_chains, n_seqs * (1 + g.C));
   g.out_tokens = c->gen_out; g.iter_log = c->gen_log; g.max_iters = D.max_ctx;
+  if (want_traj) {
+    g.traj = stats->traj;
+    g.traj_cap = stats->traj_cap;
+    g.traj_rows = stats->traj_rows;
+    g.traj_count = c->traj_count;
+    CK(cudaMemsetAsync(c->traj_count, 0, 4, c->st));
+  }
   CK(launch_gen_init(g, c->gen_state, c->gen_q0, c->seq_len, c->gen_plast, c->tok, c->pos, c->chains, c->n_chains,
                      c->res_dev, c->err, c->st));
   c->launches += 1;
@@ -861,6 +872,7 @@ jf_status generate_impl(jf_ctx* c, int n_seqs, const int32_t* const* h_prompts, 
   if (stats) {
     stats->iterations = iters;
     stats->kernel_launches = c->launches - launches0;
+    stats->traj_iters = want_traj ? std::min(iters, stats->traj_cap) : 0;
     float a = 0.f, d2 = 0.f;
     cudaEventElapsedTime(&a, e0, e1);
     cudaEventElapsedTime(&d2, e1, e2);
@@ -976,6 +988,7 @@ jf_status jf_create(const jf_model_config* model, const jf_runtime_config* rt, j
   c->gen_log = at<int>(c, O.gen_log);
   c->gen_q0 = at<int>(c, O.gen_q0);
   c->gen_plast = at<int>(c, O.gen_plast);
+  c->traj_count = at<int>(c, O.traj_count);
   c->res_dev = at<IterResult>(c, O.res);
   c->sb_dev = at<StepBlocks>(c, O.step_blocks);
   c->sres_dev = at<StepResult>(c, O.step_res);

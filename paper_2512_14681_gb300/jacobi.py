@@ -63,6 +63,20 @@ class GenOut:
     decode_ms: float
     kernel_launches: int = 0
     iter_ms: np.ndarray | None = None  # [iterations] device time of each iteration's graph replay
+    traj_iters: int = 0                # iterations recorded into the trajectory buffer
+
+
+def trajectory_records(buf, n_iters: int, traj_rows: int):
+    """Split a trajectory buffer written by jf_generate (see jf_gen_stats in include/jf.h) into one
+    dict per recorded iteration: M, it, and per row seq, kind, pos, token, pred (numpy int32)."""
+    a = buf.cpu().numpy() if hasattr(buf, "cpu") else np.asarray(buf)
+    a = a.reshape(-1)[: n_iters * (2 + 5 * traj_rows)].reshape(n_iters, 2 + 5 * traj_rows)
+    out = []
+    for rec in a:
+        M = int(rec[0])
+        f = [rec[2 + j * traj_rows: 2 + j * traj_rows + M] for j in range(5)]
+        out.append(dict(M=M, it=int(rec[1]), seq=f[0], kind=f[1], pos=f[2], token=f[3], pred=f[4]))
+    return out
 
 
 def model_config(shape: ModelShape) -> J.ModelConfig:
@@ -168,8 +182,9 @@ class Context:
         return logits, hidden, am
 
     # -- generation --------------------------------------------------------------------
-    def generate(self, prompts, gen: Gen, truth=None, log_cap: int = 4096) -> GenOut:
-        """Host buffers in and out (jf_generate)."""
+    def generate(self, prompts, gen: Gen, truth=None, log_cap: int = 4096, traj=None, traj_rows: int = 0) -> GenOut:
+        """Host buffers in and out (jf_generate). traj: optional device int32 tensor of
+        cap * (2 + 5 * traj_rows) elements that receives the Jacobi trajectory records."""
         ps = [np.ascontiguousarray(p, dtype=np.int32) for p in prompts]
         n = len(ps)
         arr = (C.POINTER(C.c_int32) * n)(*[_i32p(p) for p in ps])
@@ -185,10 +200,15 @@ class Context:
         rows = np.zeros(log_cap, dtype=np.int32)
         ims = np.zeros(max(log_cap, 1), dtype=np.float32)
         st = J.GenStats(0, _i32p(acc), _i32p(rows), log_cap, 0.0, 0.0, 0, _f32p(ims) if log_cap > 0 else None)
+        if traj is not None:
+            st.traj = traj.data_ptr()
+            st.traj_rows = traj_rows
+            st.traj_cap = traj.numel() // (2 + 5 * traj_rows)
         self._c(self.lib.jf_generate(self.h, n, arr, _i32p(lens), C.byref(gp), _i32p(out), C.byref(st)))
         it = st.iterations
         k = min(it, log_cap)
-        return GenOut(out, acc[:k], rows[:k], it, st.prefill_ms, st.decode_ms, st.kernel_launches, ims[:k])
+        return GenOut(out, acc[:k], rows[:k], it, st.prefill_ms, st.decode_ms, st.kernel_launches, ims[:k],
+                      st.traj_iters)
 
     def generate_device(self, d_prompts, prompt_lens, gen: Gen, d_out, d_truth=None, truth_len=0,
                         log_cap: int = 0):

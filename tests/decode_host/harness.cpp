@@ -30,6 +30,8 @@ int scripted_inject(const jf::GenCfg& g, int seq, int x, int P0, int it, int* er
 }  // namespace jf_host
 
 namespace {
+std::vector<int> traj_buf;
+int traj_counter = 0;
 jf::GenCfg G;
 std::vector<int> state, tok, pos, out_tokens, iter_log, truth;
 std::vector<jf::Chain> chains;
@@ -67,6 +69,22 @@ int hd_setup(int n, int K, int s_spawn, int pool_size, int Gn, int C, int mode, 
   jf_host::script.clear();
   err_word = 0;
   return 0;
+}
+
+// Trajectory record of every iteration (cap iterations of `rows` rows; cap 0 = off); call after hd_setup.
+void hd_traj(int cap, int rows) {
+  traj_buf.assign((size_t)(cap > 0 ? cap : 1) * (2 + 5 * (size_t)rows), -9);
+  traj_counter = 0;
+  G.traj = cap > 0 ? traj_buf.data() : nullptr;
+  G.traj_cap = cap;
+  G.traj_rows = rows;
+  G.traj_count = &traj_counter;
+}
+
+// Copies the trajectory buffer; returns the number of iterations recorded.
+int hd_traj_view(int* out) {
+  for (size_t i = 0; i < traj_buf.size(); ++i) out[i] = traj_buf[i];
+  return traj_counter;
 }
 
 // count < 0: the kernels' own injection rule; else (pos[i], it[i]) -> tok[i], truth elsewhere.

@@ -38,9 +38,10 @@ def _p(a):
     return a.ctypes.data_as(ctypes.POINTER(ctypes.c_int))
 
 
-def run_device(hd, pr, prompts, truths, stationary, V, script=None, wrong=wrong_const):
+def run_device(hd, pr, prompts, truths, stationary, V, script=None, wrong=wrong_const, traj_out=None):
     """Drive the host-compiled state machine with toy predictions. Returns per sequence the list of
-    its iterations (rows M, committed count k, winner, output tokens) and its generated tokens."""
+    its iterations (rows M, committed count k, winner, output tokens) and its generated tokens.
+    traj_out (a list): the trajectory record is switched on and its iterations appended there."""
     ns = len(prompts)
     if pr.mode == "ar":
         n, K, mode, pool, C = 1, 1, 1, 0, 0
@@ -62,6 +63,9 @@ def run_device(hd, pr, prompts, truths, stationary, V, script=None, wrong=wrong_
     max_ctx = max(len(p) for p in prompts) + pr.max_new + K * n + G + 8
     assert hd.hd_setup(n, K, s_spawn, pool, G, C, mode, init, T, pr.seed, pr.max_new, pr.eos_id, V, ns,
                        _p(truth_arr), truth_len, max_rows, max_chains, max_ctx) == 0
+    traj_cap = 4 * (pr.max_new + 4)
+    if traj_out is not None:
+        hd.hd_traj(traj_cap, max_rows)
     if script is None:
         hd.hd_script(-1, None, None, None)
     else:
@@ -120,6 +124,12 @@ def run_device(hd, pr, prompts, truths, stationary, V, script=None, wrong=wrong_
     else:
         raise AssertionError("decoding did not terminate")
     assert all(done)
+    if traj_out is not None:
+        buf = np.zeros(traj_cap * (2 + 5 * max_rows), dtype=np.int32)
+        n_rec = hd.hd_traj_view(_p(buf))
+        from paper_2512_14681_gb300.jacobi import trajectory_records
+
+        traj_out += trajectory_records(buf, min(n_rec, traj_cap), max_rows)
     return recs, [[int(t) for t in out[b, :nout[b]]] for b in range(ns)]
 
 
@@ -250,7 +260,8 @@ def test_device_state_machine_equals_oracle_loop(hd, case_seed, monkeypatch):
     def wrong(x, t):
         return (3 * t + x + shift) % V
 
-    recs, toks = run_device(hd, pr, prompts, truths, stationary, V, wrong=wrong)
+    traj = []
+    recs, toks = run_device(hd, pr, prompts, truths, stationary, V, wrong=wrong, traj_out=traj)
     for b in range(ns):
         calls = []
         want = run_oracle(pr, prompts[b], truths[b], stationary[b], V, monkeypatch, wrong, calls)
@@ -261,6 +272,15 @@ def test_device_state_machine_equals_oracle_loop(hd, case_seed, monkeypatch):
             assert (have["M"], have["k"], have["winner"]) == (it.M, it.k, it.winner), f"seq {b} iteration {i}: {pr}"
             assert have["fwd"] == _segments(*fwds[i][:3]), f"seq {b} iteration {i}: rows of the forward differ: {pr}"
             assert _tree_equals_chains(*fwds[i]), f"seq {b} iteration {i}: tree mask != chains: {pr}"
+            # the trajectory record of this iteration: this sequence's rows, as the oracle's loop built them
+            tr = traj[i]
+            mine = tr["seq"] == b
+            got = {k: [int(v) for v in tr[src][mine]] for k, src in
+                   (("tokens", "token"), ("pos", "pos"), ("pred", "pred"), ("kind", "kind"))}
+            assert got == {k: [int(v) for v in it.rows[k]] for k in got}, f"seq {b} iteration {i}: trajectory: {pr}"
+    # every recorded row belongs to a live sequence, and the record holds one entry per iteration
+    assert len(traj) == max(len(r) for r in recs)
+    assert all(np.all(t["seq"] >= 0) and t["M"] == int(sum(np.sum(t["seq"] == b) for b in range(ns))) for t in traj)
 
 
 def test_step_mode_verification(hd):

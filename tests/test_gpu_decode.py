@@ -163,3 +163,36 @@ def test_eos_and_device_buffers(setup):
     ctx.generate_device(d_prompt, [prompt.size], Gen(block_size=8, max_new=40), d_out)
     host = ctx.generate([prompt], Gen(block_size=8, max_new=40)).tokens[0]
     assert np.array_equal(d_out.cpu().numpy()[0], host)
+
+
+@pytest.mark.parametrize("shape", [I.TINY_F32, I.SMALL_BF16], ids=lambda s: s.name)
+def test_paper_inference_configuration_full_n(shape):
+    """The paper's inference configuration for its method (Sec. 4.3 / App. E: K = 2 blocks of
+    n = 64, spawn ratio r = 0.85, 4 verified n-grams of 64 tokens; up to 384 rows in flight) at its
+    full block size, with injected drafts: tokens and per-iteration counts against the oracle."""
+    need_gpu()
+    from paper_2512_14681_gb300.jacobi import Context, Gen
+
+    kw = dict(block_size=64, n_blocks=2, spawn_ratio=0.85, pool_size=64, cand_per_iter=4, init="inject",
+              inject_p=0.3, seed=8)
+    max_new = 192
+    ctx = Context(shape, max_seqs=1, max_ctx=1024, max_rows=384)
+    try:
+        ctx.init_random_weights(I.WEIGHT_SEED, I.WEIGHT_STD)
+        model = O.Model(O.ModelConfig(**shape.oracle_kwargs())).init_random(I.WEIGHT_SEED, I.WEIGHT_STD)
+        prompt = I.prompt_tokens(shape.vocab, 48, seed=I.PROMPT_SEED)
+        truth = OJ.generate_ar(model, prompt, max_new + 2 * 64 + 64 + 1)
+        rows = []
+
+        def run_oracle(p, n_new, offset):
+            return OJ.generate_jacobi(model, p, OJ.GenParams(max_new=n_new, **kw), truth=truth.tokens[offset:])
+
+        def run_gpu(p, n_new, offset):
+            out = ctx.generate([p], Gen(max_new=n_new, **kw), truth=np.array([truth.tokens[offset:]], dtype=np.int32))
+            rows.extend(out.rows.tolist())
+            return out.tokens[0], out.counts[:, 0]
+
+        compare_with_resync(run_gpu, run_oracle, prompt, max_new, shape.bf16, max_flags=2)
+        assert max(rows) > 128  # candidates were verified beside the blocks
+    finally:
+        ctx.close()

@@ -51,6 +51,8 @@ def test_decoding_loop_matches_hand_derived_trace(path, monkeypatch):
     for i, (rec, want) in enumerate(zip(got.iters, spec["iters"])):
         have = dict(M=rec.M, k=rec.k, winner=rec.winner, k_ra=rec.k_ra, k_cand=list(rec.k_cand),
                     pseudo=list(rec.pseudo), committed=list(rec.committed))
+        if "rows" in want:  # the forward's rows: trajectory point, positions, predictions, kinds
+            have["rows"] = {k: [int(x) for x in rec.rows[k]] for k in ("tokens", "pos", "pred", "kind")}
         assert have == want, f"iteration {i}"
     assert got.tokens == spec["tokens"]
     # every scripted corruption was drawn (an entry the loop never asked for is a typo in the script)

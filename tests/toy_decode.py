@@ -52,6 +52,13 @@ def parse(path):
                 at, tok = item.split("=")
                 pos, it = at.split("@")
                 spec["corrupt"][(int(pos), int(it))] = int(tok)
+        elif head == "rows":
+            # the rows of the preceding iteration's forward: tokens, positions, predictions, kinds
+            rows = {}
+            for item in rest.split():
+                k, v = item.split("=")
+                rows[k] = _ints(v)
+            spec["iters"][-1]["rows"] = rows
         elif head == "iter":
             rec = {}
             for item in rest.split():

@@ -154,6 +154,17 @@ typedef struct {
   int max_new, eos_id;
   const int32_t* truth;
   int truth_len;
+  /* Serving several sequences at once (all optional; NULL / 0 = off). block_sizes (HOST [n_seqs]):
+   * block size n_b of sequence b (1 .. block_size, which is then the largest); its spawn threshold
+   * is ceil(spawn_ratio * n_b); ignored in JF_MODE_AR. join_iters (HOST [n_seqs]): 0 = the sequence
+   * is prefilled before the first iteration; j > 0 = it joins at forward j: its prompt is prefilled
+   * inside the decode iterations, prefill_chunk rows (default 64) per forward beside the running
+   * sequences' Jacobi rows, and its decoding starts after its last chunk (at once if no other
+   * sequence has rows left). max_rows must hold every sequence's rows at once (a joining sequence
+   * counts max(its decode rows, prefill_chunk)). */
+  const int32_t* block_sizes;
+  const int32_t* join_iters;
+  int prefill_chunk;
 } jf_gen_params;
 
 /* Statistics of one generation. accepted (optional caller buffer [accepted_cap][n_seqs]):

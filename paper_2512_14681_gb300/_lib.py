@@ -56,7 +56,8 @@ class GenParams(C.Structure):
     _fields_ = [("block_size", C.c_int), ("n_blocks", C.c_int), ("spawn_ratio", C.c_double),
                 ("pool_size", C.c_int), ("ngram_len", C.c_int), ("cand_per_iter", C.c_int), ("mode", C.c_int),
                 ("init", C.c_int), ("inject_p", C.c_float), ("seed", C.c_uint64), ("max_new", C.c_int),
-                ("eos_id", C.c_int), ("truth", C.c_void_p), ("truth_len", C.c_int)]
+                ("eos_id", C.c_int), ("truth", C.c_void_p), ("truth_len", C.c_int), ("block_sizes", C.c_void_p),
+                ("join_iters", C.c_void_p), ("prefill_chunk", C.c_int)]
 
 
 class GenStats(C.Structure):

@@ -46,35 +46,90 @@ __device__ __forceinline__ int sentinel(int x) { return -(x + 2); }
 
 // thread 0: append pseudo-active blocks while fewer than K are active and the newest block has at
 // least s = ceil(r n) accepted tokens.
+// Block b of a sequence keeps its n tokens at S[L.blk_tok + b * g.n ..] (g.n: the largest block size).
 __device__ void spawn_blocks(const GenCfg& g, const SeqLayout& L, int* S) {
   if (g.K <= 1) return;
-  const int n = g.n;
+  const int n = S[H_N], nst = g.n;
   while (S[H_NBLK] < g.K) {
     const int last = S[H_NBLK] - 1;
     const int start_last = S[L.blk_start + last];
     const int progress = (last == 0) ? (S[H_P] - start_last) : S[L.blk_na + last];
-    if (progress < g.s_spawn) break;
+    if (progress < S[H_SSPAWN]) break;
     const int nb = last + 1;
     const int start = start_last + n;
-    const int prev_tok = (last == 0) ? S[L.blk_tok + S[H_RA_LEN] - 1] : S[L.blk_tok + last * n + n - 1];
+    const int prev_tok = (last == 0) ? S[L.blk_tok + S[H_RA_LEN] - 1] : S[L.blk_tok + last * nst + n - 1];
     S[L.blk_start + nb] = start;
     S[L.blk_na + nb] = 0;
-    for (int j = 0; j < n; ++j) S[L.blk_tok + nb * n + j] = (g.init == GI_INJECT) ? sentinel(start + j) : prev_tok;
+    for (int j = 0; j < n; ++j) S[L.blk_tok + nb * nst + j] = (g.init == GI_INJECT) ? sentinel(start + j) : prev_tok;
     S[H_NBLK] = nb + 1;
   }
+}
+
+// thread 0: first drafts of a sequence whose prompt (P tokens) is committed: the RA block
+// [q0, fill ...] of its block size, pseudo blocks spawned, empty pool.
+__device__ void init_decode(const GenCfg& g, const SeqLayout& L, int* S, int P, int q0, int prompt_last) {
+  const int n = S[H_N];
+  S[H_PHASE] = PH_DECODE;
+  S[H_P] = P;
+  S[H_P0] = P;
+  S[H_Q0] = q0;
+  S[H_LAST] = prompt_last;
+  S[H_NBLK] = 1;
+  S[L.blk_start] = P;
+  S[H_RA_LEN] = n;
+  S[L.blk_tok] = q0;
+  for (int j = 1; j < n; ++j) S[L.blk_tok + j] = (g.init == GI_INJECT) ? sentinel(P + j) : prompt_last;
+  spawn_blocks(g, L, S);
+}
+
+// all threads: the rows of the next prefill chunk of a sequence that joined late -- its next
+// prompt tokens at the next positions, one causal chain over the committed prefix.
+__device__ void finalize_prefill(const GenCfg& g, int* S, int seq, int row_off, int* tok, int* pos, Chain* chains,
+                                 int* s_nch, int* s_rows, int* err) {
+  const int P = S[H_P], pf = S[H_PF], plen = S[H_PLEN], poff = S[H_POFF];
+  const int c = g.prefill_chunk < plen - pf ? g.prefill_chunk : plen - pf;
+  const bool fits = c >= 1 && P == pf && row_off + c <= g.max_rows && *s_nch + 1 <= g.max_chains && P + c <= g.max_ctx;
+  if (!fits) {
+    if (threadIdx.x == 0) {
+      jf_set_error(err, JF_DERR_BOUNDS);
+      S[H_DONE] = 1;
+      *s_rows = 0;
+    }
+    __syncthreads();
+    return;
+  }
+  for (int j = threadIdx.x; j < c; j += blockDim.x) {
+    tok[row_off + j] = g.prompts[poff + pf + j];
+    pos[row_off + j] = P + j;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    S[H_MAIN_ROW0] = row_off;
+    S[H_MAIN_LEN] = c;
+    S[H_RA_LEN] = c;
+    S[H_NCAND] = 0;
+    chains[*s_nch] = Chain{seq, row_off, c, P};
+    *s_nch += 1;
+    *s_rows = c;
+  }
+  __syncthreads();
 }
 
 // all threads: resolve injection sentinels, then write this sequence's rows of the next forward
 // starting at row_off (thread 0 returns the row count through *s_rows).
 __device__ void finalize_seq(const GenCfg& g, const SeqLayout& L, int* S, int seq, int row_off, int* tok, int* pos,
                              Chain* chains, int* s_nch, int* s_rows, int* err) {
-  const int n = g.n;
+  if (S[H_PHASE] == PH_PREFILL) {
+    finalize_prefill(g, S, seq, row_off, tok, pos, chains, s_nch, s_rows, err);
+    return;
+  }
+  const int n = S[H_N], nst = g.n;
   const int nblk = S[H_NBLK], Lra = S[H_RA_LEN];
   const int it = S[H_IT], P0 = S[H_P0];
   // sentinels can only be in the RA draft and the pseudo blocks
   const int nslots = Lra + (nblk - 1) * n;
   for (int i = threadIdx.x; i < nslots; i += blockDim.x) {
-    int* slot = (i < Lra) ? &S[L.blk_tok + i] : &S[L.blk_tok + n + (i - Lra)];
+    int* slot = (i < Lra) ? &S[L.blk_tok + i] : &S[L.blk_tok + (1 + (i - Lra) / n) * nst + (i - Lra) % n];
     const int v = *slot;
     if (v < 0) *slot = inject_token(g, seq, -v - 2, P0, it, err);
   }
@@ -101,7 +156,7 @@ __device__ void finalize_seq(const GenCfg& g, const SeqLayout& L, int* S, int se
       pos[row_off + i] = P + i;
     } else {
       const int bi = 1 + (i - Lra) / n, j = (i - Lra) % n;
-      tok[row_off + i] = S[L.blk_tok + bi * n + j];
+      tok[row_off + i] = S[L.blk_tok + bi * nst + j];
       pos[row_off + i] = S[L.blk_start + bi] + j;
     }
   }
@@ -132,7 +187,44 @@ __device__ void finalize_seq(const GenCfg& g, const SeqLayout& L, int* S, int se
   __syncthreads();
 }
 
-// Initial drafts after prefill: RA block [q0, fill...], pseudo blocks spawned, empty pool.
+// thread 0: the first waiting sequence (not done) starts its prefill now; -1 if there is none.
+__device__ int first_waiting(const GenCfg& g, const int* state) {
+  for (int b = 0; b < g.n_seqs; ++b) {
+    const int* S = state + (size_t)b * g.state_stride;
+    if (!S[H_DONE] && S[H_PHASE] == PH_WAIT) return b;
+  }
+  return -1;
+}
+
+// all threads: when the next forward would have no rows but a sequence still waits to join, that
+// sequence starts its prefill in it (a later join iteration cannot be reached without a forward).
+__device__ void join_if_idle(const GenCfg& g, int* state, int* S, int* row_off, int* tok, int* pos, Chain* chains,
+                             int* s_nch, int* s_rows, int* err, IterResult* res) {
+  __shared__ int s_b;
+  if (threadIdx.x == 0) s_b = (*row_off == 0) ? first_waiting(g, state) : -1;
+  __syncthreads();
+  const int b = s_b;
+  if (b < 0) return;
+  int* Sg = state + (size_t)b * g.state_stride;
+  for (int i = threadIdx.x; i < g.state_stride; i += blockDim.x) S[i] = Sg[i];
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    S[H_PHASE] = PH_PREFILL;
+    S[H_PF] = 0;
+    S[H_P] = 0;
+  }
+  __syncthreads();
+  const SeqLayout L = seq_layout(g.n, g.K, g.C, g.G, g.pool_size);
+  finalize_seq(g, L, S, b, *row_off, tok, pos, chains, s_nch, s_rows, err);
+  *row_off += *s_rows;
+  for (int i = threadIdx.x; i < g.state_stride; i += blockDim.x) Sg[i] = S[i];
+  if (threadIdx.x == 0) res->P[b] = S[H_P];
+  __syncthreads();
+}
+
+// Initial drafts after prefill: RA block [q0, fill...], pseudo blocks spawned, empty pool. A
+// sequence with a join iteration j > 0 waits (no rows) until forward j, where its chunked prefill
+// starts.
 __global__ void k_gen_init(const GenCfg g, int* state, const int* q0, const int* seq_len, const int* prompt_last,
                            int* tok, int* pos, Chain* chains, int* n_chains_dev, IterResult* res, int* err) {
   extern __shared__ int S[];
@@ -145,21 +237,25 @@ __global__ void k_gen_init(const GenCfg g, int* state, const int* q0, const int*
     for (int i = threadIdx.x; i < g.state_stride; i += blockDim.x) S[i] = 0;
     __syncthreads();
     if (threadIdx.x == 0) {
-      const int P = seq_len[b];
-      S[H_P] = P;
-      S[H_P0] = P;
-      S[H_Q0] = q0[b];
-      S[H_LAST] = prompt_last[b];
-      S[H_NBLK] = 1;
-      S[L.blk_start] = P;
-      S[H_RA_LEN] = g.n;
-      S[L.blk_tok] = q0[b];
-      for (int j = 1; j < g.n; ++j) S[L.blk_tok + j] = (g.init == GI_INJECT) ? sentinel(P + j) : prompt_last[b];
-      spawn_blocks(g, L, S);
+      const int* sp = g.seq_params + (size_t)b * kSeqParams;
+      S[H_N] = sp[SP_N];
+      S[H_SSPAWN] = sp[SP_SSPAWN];
+      S[H_JOIN] = sp[SP_JOIN];
+      S[H_POFF] = sp[SP_POFF];
+      S[H_PLEN] = sp[SP_PLEN];
+      s_rows = 0;
+      if (sp[SP_JOIN] <= 0) {
+        S[H_PF] = sp[SP_PLEN];
+        init_decode(g, L, S, seq_len[b], q0[b], prompt_last[b]);
+      } else {
+        S[H_PHASE] = PH_WAIT;
+      }
     }
     __syncthreads();
-    finalize_seq(g, L, S, b, row_off, tok, pos, chains, &s_nch, &s_rows, err);
-    row_off += s_rows;
+    if (S[H_PHASE] != PH_WAIT) {
+      finalize_seq(g, L, S, b, row_off, tok, pos, chains, &s_nch, &s_rows, err);
+      row_off += s_rows;
+    }
     for (int i = threadIdx.x; i < g.state_stride; i += blockDim.x) state[(size_t)b * g.state_stride + i] = S[i];
     if (threadIdx.x == 0) {
       res->k[b] = 0;
@@ -169,6 +265,7 @@ __global__ void k_gen_init(const GenCfg g, int* state, const int* q0, const int*
     }
     __syncthreads();
   }
+  join_if_idle(g, state, S, &row_off, tok, pos, chains, &s_nch, &s_rows, err, res);
   if (threadIdx.x == 0) {
     *n_chains_dev = s_nch;
     res->next_M = row_off;
@@ -207,12 +304,14 @@ __device__ void record_trajectory(const GenCfg& g, const SeqLayout& L, const int
     for (int b = 0; b < g.n_seqs; ++b) {
       const int* S = state + (size_t)b * g.state_stride;
       if (S[H_DONE]) continue;  // a finished sequence has no rows in this forward
+      if (S[H_PHASE] == PH_WAIT) continue;  // nor does one still waiting to join
       const int mr0 = S[H_MAIN_ROW0], mlen = S[H_MAIN_LEN], lra = S[H_RA_LEN];
+      const bool prefill = S[H_PHASE] == PH_PREFILL;
       for (int r = threadIdx.x; r < mlen; r += blockDim.x) {
         const int row = mr0 + r;
         if (row >= 0 && row < Mr) {
           rec[2 + row] = b;
-          rec[2 + R + row] = r < lra ? 0 : 1;
+          rec[2 + R + row] = prefill ? 3 : (r < lra ? 0 : 1);
         }
       }
       const int nc = S[H_NCAND];
@@ -246,7 +345,7 @@ __global__ void k_gen_accept(const GenCfg g, int* state, const int* gpred, int M
   if (threadIdx.x == 0) s_nch = 0;
   __syncthreads();
   if (g.traj) record_trajectory(g, L, state, gp, M_cur, tok, pos);
-  const int n = g.n, G = g.G;
+  const int nst = g.n, G = g.G;
   int row_off = 0;
   int all_done = 1;
   for (int b = 0; b < g.n_seqs; ++b) {
@@ -256,7 +355,27 @@ __global__ void k_gen_accept(const GenCfg g, int* state, const int* gpred, int M
     const bool was_done = S[H_DONE] != 0;
     if (threadIdx.x == 0) {
       commit[b] = CommitInfo{0, 0, S[H_P]};
-      if (!was_done) {
+      const int git = S[H_GIT];
+      S[H_GIT] = git + 1;
+      if (!was_done && S[H_PHASE] == PH_WAIT) {
+        // a late sequence joins: its first prefill chunk rides in the next forward
+        if (git + 1 >= S[H_JOIN]) {
+          S[H_PHASE] = PH_PREFILL;
+          S[H_PF] = 0;
+          S[H_P] = 0;
+        }
+      } else if (!was_done && S[H_PHASE] == PH_PREFILL) {
+        // a prefill chunk ran: all its rows are committed; after the last one, decoding starts
+        const int mr0 = S[H_MAIN_ROW0], c = S[H_MAIN_LEN], P = S[H_P];
+        commit[b] = CommitInfo{mr0, c, P};
+        S[H_PF] += c;
+        S[H_P] = P + c;
+        S[H_LAST_K] = 0;
+        S[H_WINNER] = 0;
+        if (S[H_PF] >= S[H_PLEN])
+          init_decode(g, L, S, P + c, gp[mr0 + c - 1], g.prompts[S[H_POFF] + S[H_PLEN] - 1]);
+      } else if (!was_done) {
+        const int n = S[H_N];
         const int P = S[H_P], Lra = S[H_RA_LEN], mr0 = S[H_MAIN_ROW0], mlen = S[H_MAIN_LEN];
         const int nblk = S[H_NBLK];
         int* ra = S + L.blk_tok;
@@ -304,7 +423,7 @@ __global__ void k_gen_accept(const GenCfg g, int* state, const int* gpred, int M
             const int idx = k_ra + j;
             int tv;
             if (idx < mlen) {
-              tv = (idx < Lra) ? ra[idx] : S[L.blk_tok + (1 + (idx - Lra) / n) * n + (idx - Lra) % n];
+              tv = (idx < Lra) ? ra[idx] : S[L.blk_tok + (1 + (idx - Lra) / n) * nst + (idx - Lra) % n];
             } else {
               tv = prev;
             }
@@ -316,7 +435,7 @@ __global__ void k_gen_accept(const GenCfg g, int* state, const int* gpred, int M
         for (int bi = 1; bi < nblk; ++bi) {
           const int start = S[L.blk_start + bi];
           int na = S[L.blk_na + bi];
-          int* bt = S + L.blk_tok + bi * n;
+          int* bt = S + L.blk_tok + bi * nst;
           while (na < n && bt[na] == gp[mr0 + (start + na - 1 - P)]) ++na;
           S[L.blk_na + bi] = na;
           for (int x = start + na; x < start + n; ++x)
@@ -349,13 +468,13 @@ __global__ void k_gen_accept(const GenCfg g, int* state, const int* gpred, int M
           for (int x = Pn + 1; x < Pn + n; ++x) ra[x - Pn] = (g.init == GI_INJECT) ? sentinel(x) : tail_pred(x, last);
         } else if (Pn >= ra_start + n) {
           if (nblk > 1) {
-            for (int j = 0; j < n; ++j) ra[j] = S[L.blk_tok + n + j];
+            for (int j = 0; j < n; ++j) ra[j] = S[L.blk_tok + nst + j];
             ra[0] = new_q0;
             S[L.blk_start] = S[L.blk_start + 1];
             for (int bi = 1; bi + 1 < nblk; ++bi) {
               S[L.blk_start + bi] = S[L.blk_start + bi + 1];
               S[L.blk_na + bi] = S[L.blk_na + bi + 1];
-              for (int j = 0; j < n; ++j) S[L.blk_tok + bi * n + j] = S[L.blk_tok + (bi + 1) * n + j];
+              for (int j = 0; j < n; ++j) S[L.blk_tok + bi * nst + j] = S[L.blk_tok + (bi + 1) * nst + j];
             }
             S[H_NBLK] = nblk - 1;
           } else {
@@ -393,7 +512,7 @@ __global__ void k_gen_accept(const GenCfg g, int* state, const int* gpred, int M
       }
     }
     __syncthreads();
-    if (!S[H_DONE]) {
+    if (!S[H_DONE] && S[H_PHASE] != PH_WAIT) {
       finalize_seq(g, L, S, b, row_off, tok, pos, chains, &s_nch, &s_rows, err);
       row_off += s_rows;
     }
@@ -407,6 +526,7 @@ __global__ void k_gen_accept(const GenCfg g, int* state, const int* gpred, int M
     }
     __syncthreads();
   }
+  join_if_idle(g, state, S, &row_off, tok, pos, chains, &s_nch, &s_rows, err, res);
   if (threadIdx.x == 0) {
     *n_chains_dev = s_nch;
     res->next_M = row_off;

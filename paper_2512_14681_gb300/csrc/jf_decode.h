@@ -10,7 +10,7 @@ enum GenMode : int { GM_BLOCK = 0, GM_WINDOW = 1 };
 enum GenInit : int { GI_REPEAT = 0, GI_INJECT = 1 };
 
 struct GenCfg {
-  int n, K, s_spawn, pool_size, G, C, mode, init;
+  int n, K, s_spawn, pool_size, G, C, mode, init;  // n: the largest block size (state slot stride)
   unsigned long long T, seed;
   int max_new, eos, V, n_seqs;
   const int* truth;       // [n_seqs][truth_stride] greedy continuation from the prompt end
@@ -26,12 +26,23 @@ struct GenCfg {
   int* traj;
   int traj_cap, traj_rows;
   int* traj_count;        // device counter of recorded iterations (zeroed by the host per call)
+  // Per sequence [n_seqs][kSeqParams]: block size, spawn threshold ceil(r n), join iteration (0 =
+  // prefilled before the first iteration; j > 0 = its prompt is prefilled inside the iterations from
+  // forward j on, prefill_chunk rows per forward), prompt offset in `prompts`, prompt length.
+  const int* seq_params;
+  const int* prompts;     // prompts of the sequences that join later (device)
+  int prefill_chunk;
 };
+constexpr int kSeqParams = 5;
+enum SeqParam : int { SP_N = 0, SP_SSPAWN, SP_JOIN, SP_POFF, SP_PLEN };
+// Phase of a sequence: Jacobi decoding, waiting to join, or prefilling its prompt in chunks.
+enum SeqPhase : int { PH_DECODE = 0, PH_WAIT = 1, PH_PREFILL = 2 };
 
 // Layout of one sequence's state (ints). Header fields first.
 enum SeqHdr : int {
   H_P = 0, H_Q0, H_NOUT, H_DONE, H_IT, H_LAST, H_NBLK, H_RA_START, H_RA_LEN, H_NCAND, H_POOL_N, H_POOL_HEAD,
-  H_P0, H_MAIN_ROW0, H_MAIN_LEN, H_LAST_K, H_WINNER, H_COUNT
+  H_P0, H_MAIN_ROW0, H_MAIN_LEN, H_LAST_K, H_WINNER, H_N, H_SSPAWN, H_PHASE, H_JOIN, H_PF, H_PLEN, H_POFF, H_GIT,
+  H_COUNT
 };
 
 struct SeqLayout {

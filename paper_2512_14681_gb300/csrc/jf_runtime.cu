@@ -111,7 +111,8 @@ struct Offsets {
   size_t tok, pos, gpred, top2, chains, n_chains, attn_xchg;
   size_t gemm_ws, gemm_counter, am_v1, am_i1, am_v2, am_counter;
   size_t logits, err, traj_count;
-  size_t gen_state, gen_out, gen_truth, gen_log, gen_q0, gen_plast, res, step_blocks, step_res, committed;
+  size_t gen_state, gen_out, gen_truth, gen_log, gen_q0, gen_plast, gen_prompt, gen_seqp, res, step_blocks, step_res,
+      committed;
   size_t gemm_ws_bytes;
   size_t total;
 };
@@ -228,6 +229,8 @@ Offsets plan_offsets(const Dims& D) {
   o.gen_log = p.take((size_t)D.max_ctx * D.S * 4);
   o.gen_q0 = p.take((size_t)D.S * 4);
   o.gen_plast = p.take((size_t)D.S * 4);
+  o.gen_prompt = p.take((size_t)D.S * D.max_ctx * 4);
+  o.gen_seqp = p.take((size_t)D.S * kSeqParams * 4);
   o.res = p.take(sizeof(IterResult));
   o.step_blocks = p.take(sizeof(StepBlocks));
   o.step_res = p.take(sizeof(StepResult));
@@ -293,7 +296,7 @@ struct jf_ctx {
   int *am_i1, *am_counter;
   float* logits;
   int* err;
-  int *gen_state, *gen_out, *gen_truth, *gen_log, *gen_q0, *gen_plast, *traj_count;
+  int *gen_state, *gen_out, *gen_truth, *gen_log, *gen_q0, *gen_plast, *gen_prompt, *gen_seqp, *traj_count;
   IterResult* res_dev;
   StepBlocks* sb_dev;
   StepResult* sres_dev;
@@ -718,7 +721,8 @@ jf_status generate_impl(jf_ctx* c, int n_seqs, const int32_t* const* h_prompts, 
   if (!c->weights_ready) return fail(c, JF_ESTATE, "weights not initialised");
   if (!gp || n_seqs < 1 || n_seqs > D.S || !prompt_lens) return fail(c, JF_EINVAL, "bad n_seqs / params");
   jf_gen_params p = *gp;
-  if (p.mode == JF_MODE_AR) {
+  const bool ar = p.mode == JF_MODE_AR;
+  if (ar) {
     p.mode = JF_MODE_WINDOW;
     p.block_size = 1;
     p.n_blocks = 1;
@@ -734,8 +738,22 @@ jf_status generate_impl(jf_ctx* c, int n_seqs, const int32_t* const* h_prompts, 
   if (!(p.inject_p >= 0.f && p.inject_p <= 1.f)) return fail(c, JF_EINVAL, "inject_p must be in [0, 1]");
   const int G = p.ngram_len > 0 ? p.ngram_len : p.block_size;
   const int C = p.pool_size > 0 ? p.cand_per_iter : 0;
-  const int rows_per_seq = p.n_blocks * p.block_size + C * G;
-  if (rows_per_seq * n_seqs > D.R) return fail(c, JF_ECAPACITY, "in-flight rows exceed max_rows");
+  const int rows_per_seq = p.n_blocks * p.block_size + C * G;  // at the largest block size
+  // per-sequence block sizes (serving several requests at once) and late joins (chunked prefill
+  // inside the decode iterations)
+  const int chunk = p.prefill_chunk > 0 ? p.prefill_chunk : 64;
+  std::vector<int> nb(n_seqs, p.block_size), join(n_seqs, 0);
+  long long rows_total = 0;
+  for (int b = 0; b < n_seqs; ++b) {
+    if (p.block_sizes && !ar) nb[b] = p.block_sizes[b];
+    if (p.join_iters) join[b] = p.join_iters[b];
+    if (nb[b] < 1 || nb[b] > p.block_size) return fail(c, JF_EINVAL, "block_sizes[b] must be in 1..block_size");
+    if (join[b] < 0 || join[b] > (1 << 20)) return fail(c, JF_EINVAL, "join_iters[b] out of range");
+    const int rb = p.n_blocks * nb[b] + C * std::min(G, nb[b]);  // candidates are cut to the draft length
+    rows_total += join[b] > 0 ? std::max(rb, chunk) : rb;
+  }
+  if (chunk > D.R) return fail(c, JF_EINVAL, "prefill_chunk exceeds max_rows");
+  if (rows_total > D.R) return fail(c, JF_ECAPACITY, "in-flight rows exceed max_rows");
   if (1 + C > 5) return fail(c, JF_EINVAL, "too many candidates");
   const SeqLayout L = seq_layout(p.block_size, p.n_blocks, C, G, p.pool_size);
   if (L.total > kMaxStateInts || (size_t)(L.total + D.R) * 4 > 200 * 1024)
@@ -761,7 +779,7 @@ jf_status generate_impl(jf_ctx* c, int n_seqs, const int32_t* const* h_prompts, 
     if (s != JF_OK) return s;
   }
   const bool want_traj = stats && stats->traj;
-  if (want_traj && (stats->traj_cap < 1 || stats->traj_rows < rows_per_seq * n_seqs))
+  if (want_traj && (stats->traj_cap < 1 || stats->traj_rows < rows_total))
     return fail(c, JF_EINVAL, "trajectory buffer: traj_cap >= 1 and traj_rows >= the rows of one forward needed");
   // reset slots 0 .. n_seqs-1 and reserve their pages
   for (int b = 0; b < n_seqs; ++b) {
@@ -786,17 +804,32 @@ jf_status generate_impl(jf_ctx* c, int n_seqs, const int32_t* const* h_prompts, 
     CK(cudaEventCreate(&ev.e[4]));
   }
   CK(cudaEventRecord(e0, c->st));
-  std::vector<int> q0(n_seqs), plast(n_seqs);
-  long long off = 0;
+  std::vector<int> q0(n_seqs, 0), plast(n_seqs, 0), seqp((size_t)n_seqs * kSeqParams, 0);
+  long long off = 0, loff = 0;  // offsets in the caller's prompts and in the late prompts' buffer
   for (int b = 0; b < n_seqs; ++b) {
-    int32_t nt = -1;
-    jf_status s = prefill_impl(c, b, device_io ? nullptr : h_prompts[b], device_io ? d_prompts + off : nullptr, plen[b], &nt);
-    if (s != JF_OK) return s;
-    q0[b] = nt;
-    if (device_io) CK(cudaMemcpy(&plast[b], d_prompts + off + plen[b] - 1, 4, cudaMemcpyDeviceToHost));
-    else plast[b] = h_prompts[b][plen[b] - 1];
+    int* sp = &seqp[(size_t)b * kSeqParams];
+    sp[SP_N] = nb[b];
+    sp[SP_SSPAWN] = (int)std::ceil(p.spawn_ratio * nb[b] - 1e-12);
+    sp[SP_JOIN] = join[b];
+    sp[SP_PLEN] = plen[b];
+    if (join[b] > 0) {
+      // prefilled later, inside the decode iterations: keep its prompt on the device
+      if (loff + plen[b] > (long long)D.S * D.max_ctx) return fail(c, JF_ECAPACITY, "late prompts exceed their buffer");
+      sp[SP_POFF] = (int)loff;
+      CK(cudaMemcpyAsync(c->gen_prompt + loff, device_io ? d_prompts + off : h_prompts[b], (size_t)plen[b] * 4,
+                         device_io ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice, c->st));
+      loff += plen[b];
+    } else {
+      int32_t nt = -1;
+      jf_status s = prefill_impl(c, b, device_io ? nullptr : h_prompts[b], device_io ? d_prompts + off : nullptr, plen[b], &nt);
+      if (s != JF_OK) return s;
+      q0[b] = nt;
+      if (device_io) CK(cudaMemcpy(&plast[b], d_prompts + off + plen[b] - 1, 4, cudaMemcpyDeviceToHost));
+      else plast[b] = h_prompts[b][plen[b] - 1];
+    }
     off += plen[b];
   }
+  CK(cudaMemcpyAsync(c->gen_seqp, seqp.data(), seqp.size() * 4, cudaMemcpyHostToDevice, c->st));
   CK(cudaEventRecord(e1, c->st));
   CK(cudaMemcpyAsync(c->gen_q0, q0.data(), (size_t)n_seqs * 4, cudaMemcpyHostToDevice, c->st));
   CK(cudaMemcpyAsync(c->gen_plast, plast.data(), (size_t)n_seqs * 4, cudaMemcpyHostToDevice, c->st));
@@ -819,8 +852,11 @@ jf_status generate_impl(jf_ctx* c, int n_seqs, const int32_t* const* h_prompts, 
   g.truth_len = p.init == JF_INIT_INJECT ? p.truth_len : 0;
   g.state_stride = L.total;
   g.max_rows = D.R; g.max_chains = D.max_chains; g.max_ctx = D.max_ctx;
-  c->chains_bound = std::min(D.max_chains, n_seqs * (1 + g.C));
+  c->chains_bound = std::min(D.max_chains, n_seqs * (1 + g.C));  // a prefilling sequence has one chain
   g.out_tokens = c->gen_out; g.iter_log = c->gen_log; g.max_iters = D.max_ctx;
+  g.seq_params = c->gen_seqp;
+  g.prompts = c->gen_prompt;
+  g.prefill_chunk = chunk;
   if (want_traj) {
     g.traj = stats->traj;
     g.traj_cap = stats->traj_cap;
@@ -859,7 +895,8 @@ jf_status generate_impl(jf_ctx* c, int n_seqs, const int32_t* const* h_prompts, 
     if ((s = check_err_word(c, c->res_host->err)) != JF_OK) return s;
     done = c->res_host->all_done != 0;
     M = c->res_host->next_M;
-    if (iters > D.max_ctx) return fail(c, JF_EDEVICE, "decoding did not terminate");
+    // every forward commits a token or a prefill chunk of some sequence
+    if (iters > (long long)D.max_ctx * n_seqs + 16) return fail(c, JF_EDEVICE, "decoding did not terminate");
   }
   CK(cudaEventRecord(e2, c->st));
   if (device_io) {
@@ -989,6 +1026,8 @@ jf_status jf_create(const jf_model_config* model, const jf_runtime_config* rt, j
   c->gen_q0 = at<int>(c, O.gen_q0);
   c->gen_plast = at<int>(c, O.gen_plast);
   c->traj_count = at<int>(c, O.traj_count);
+  c->gen_prompt = at<int>(c, O.gen_prompt);
+  c->gen_seqp = at<int>(c, O.gen_seqp);
   c->res_dev = at<IterResult>(c, O.res);
   c->sb_dev = at<StepBlocks>(c, O.step_blocks);
   c->sres_dev = at<StepResult>(c, O.step_res);

@@ -44,13 +44,26 @@ class Gen:
     seed: int = 0
     max_new: int = 64
     eos_id: int = -1
+    block_sizes: tuple | None = None   # per-sequence block sizes (block_size = the largest)
+    join_iters: tuple | None = None    # per-sequence join iteration (0 = prefilled first)
+    prefill_chunk: int = 0             # rows of one in-iteration prefill chunk (0 = 64)
 
     def c_struct(self, truth_ptr=None, truth_len=0) -> J.GenParams:
         mode = {"block": J.JF_MODE_BLOCK, "window": J.JF_MODE_WINDOW, "ar": J.JF_MODE_AR}[self.mode]
         init = {"repeat": J.JF_INIT_REPEAT, "inject": J.JF_INIT_INJECT}[self.init]
-        return J.GenParams(self.block_size, self.n_blocks, self.spawn_ratio, self.pool_size, self.ngram_len,
-                           self.cand_per_iter, mode, init, self.inject_p, self.seed, self.max_new, self.eos_id,
-                           truth_ptr, truth_len)
+        gp = J.GenParams(self.block_size, self.n_blocks, self.spawn_ratio, self.pool_size, self.ngram_len,
+                         self.cand_per_iter, mode, init, self.inject_p, self.seed, self.max_new, self.eos_id,
+                         truth_ptr, truth_len)
+        # the per-sequence arrays live as long as the returned structure
+        gp._keep = []
+        for name in ("block_sizes", "join_iters"):
+            v = getattr(self, name)
+            if v is not None:
+                a = np.ascontiguousarray(v, dtype=np.int32)
+                gp._keep.append(a)
+                setattr(gp, name, a.ctypes.data)
+        gp.prefill_chunk = self.prefill_chunk
+        return gp
 
 
 @dataclass

@@ -33,7 +33,7 @@ namespace {
 std::vector<int> traj_buf;
 int traj_counter = 0;
 jf::GenCfg G;
-std::vector<int> state, tok, pos, out_tokens, iter_log, truth;
+std::vector<int> state, tok, pos, out_tokens, iter_log, truth, seqp, late_prompts;
 std::vector<jf::Chain> chains;
 std::vector<jf::CommitInfo> commit;
 jf::IterResult res;
@@ -42,9 +42,12 @@ int n_chains_dev = 0, err_word = 0;
 
 extern "C" {
 
+// seq_n / seq_spawn / join / prompts / prompt_lens: per sequence block size, spawn threshold, join
+// iteration (0 = prefilled before the first iteration) and prompt (all prompts concatenated).
 int hd_setup(int n, int K, int s_spawn, int pool_size, int Gn, int C, int mode, int init, unsigned long long T,
              unsigned long long seed, int max_new, int eos, int V, int n_seqs, const int* truth_in, int truth_len,
-             int max_rows, int max_chains, int max_ctx) {
+             int max_rows, int max_chains, int max_ctx, const int* seq_n, const int* seq_spawn, const int* join,
+             const int* prompts, const int* prompt_lens, int prefill_chunk) {
   if (n_seqs < 1 || n_seqs > jf::kMaxSeqs) return 1;
   const jf::SeqLayout L = jf::seq_layout(n, K, C, Gn, pool_size);
   G = jf::GenCfg{};
@@ -64,6 +67,22 @@ int hd_setup(int n, int K, int s_spawn, int pool_size, int Gn, int C, int mode, 
   out_tokens.assign((size_t)n_seqs * max_new, -1);
   iter_log.assign((size_t)max_ctx * n_seqs, -1);
   G.out_tokens = out_tokens.data(); G.iter_log = iter_log.data(); G.max_iters = max_ctx;
+  seqp.assign((size_t)n_seqs * jf::kSeqParams, 0);
+  late_prompts.clear();
+  for (int b = 0; b < n_seqs; ++b) {
+    int* sp = &seqp[(size_t)b * jf::kSeqParams];
+    sp[jf::SP_N] = seq_n[b];
+    sp[jf::SP_SSPAWN] = seq_spawn[b];
+    sp[jf::SP_JOIN] = join[b];
+    sp[jf::SP_POFF] = (int)late_prompts.size();
+    sp[jf::SP_PLEN] = prompt_lens[b];
+    long long off = 0;
+    for (int c = 0; c < b; ++c) off += prompt_lens[c];
+    late_prompts.insert(late_prompts.end(), prompts + off, prompts + off + prompt_lens[b]);
+  }
+  G.seq_params = seqp.data();
+  G.prompts = late_prompts.data();
+  G.prefill_chunk = prefill_chunk;
   jf_host::smem.assign((size_t)L.total + max_rows, 0);
   jf_host::use_script = false;
   jf_host::script.clear();

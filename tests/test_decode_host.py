@@ -38,16 +38,23 @@ def _p(a):
     return a.ctypes.data_as(ctypes.POINTER(ctypes.c_int))
 
 
-def run_device(hd, pr, prompts, truths, stationary, V, script=None, wrong=wrong_const, traj_out=None):
+def run_device(hd, pr, prompts, truths, stationary, V, script=None, wrong=wrong_const, traj_out=None, seq_n=None,
+               join=None, chunk=4):
     """Drive the host-compiled state machine with toy predictions. Returns per sequence the list of
-    its iterations (rows M, committed count k, winner, output tokens) and its generated tokens.
-    traj_out (a list): the trajectory record is switched on and its iterations appended there."""
+    its decoding iterations (rows M, committed count k, winner, output tokens) and its generated
+    tokens. traj_out (a list): the trajectory record is switched on and its iterations appended there.
+    seq_n: per-sequence block sizes (pr.block_size is then the largest); join: per-sequence join
+    iteration (0 = prefilled before the first iteration, else prefilled in `chunk`-row pieces inside
+    the iterations)."""
     ns = len(prompts)
     if pr.mode == "ar":
         n, K, mode, pool, C = 1, 1, 1, 0, 0
+        seq_n = None
     else:
         n, K, mode, pool = pr.block_size, pr.n_blocks, (1 if pr.mode == "window" else 0), pr.pool_size
         C = pr.cand_per_iter if pool > 0 else 0
+    seq_n = list(seq_n) if seq_n is not None else [n] * ns
+    join = list(join) if join is not None else [0] * ns
     G = pr.ngram_len or n
     init = 1 if pr.init == "inject" else 0
     s_spawn = math.ceil(pr.spawn_ratio * n - 1e-12)
@@ -58,11 +65,17 @@ def run_device(hd, pr, prompts, truths, stationary, V, script=None, wrong=wrong_
     for b in range(ns):
         if init:
             truth_arr[b] = truths[b][len(prompts[b]):len(prompts[b]) + truth_len]
-    max_rows = ns * (K * n + C * G)
+    max_rows = ns * max(K * n + C * G, chunk)
     max_chains = ns * (1 + C)
     max_ctx = max(len(p) for p in prompts) + pr.max_new + K * n + G + 8
+    sn = np.array(seq_n, dtype=np.int32)
+    ss = np.array([math.ceil(pr.spawn_ratio * x - 1e-12) for x in seq_n], dtype=np.int32)
+    jn = np.array(join, dtype=np.int32)
+    flat = np.array([t for p in prompts for t in p], dtype=np.int32)
+    plens = np.array([len(p) for p in prompts], dtype=np.int32)
     assert hd.hd_setup(n, K, s_spawn, pool, G, C, mode, init, T, pr.seed, pr.max_new, pr.eos_id, V, ns,
-                       _p(truth_arr), truth_len, max_rows, max_chains, max_ctx) == 0
+                       _p(truth_arr), truth_len, max_rows, max_chains, max_ctx, _p(sn), _p(ss), _p(jn), _p(flat),
+                       _p(plens), chunk) == 0
     traj_cap = 4 * (pr.max_new + 4)
     if traj_out is not None:
         hd.hd_traj(traj_cap, max_rows)
@@ -72,7 +85,7 @@ def run_device(hd, pr, prompts, truths, stationary, V, script=None, wrong=wrong_
         ks = sorted(script)
         cols = [np.array(c, dtype=np.int32) for c in ([k[0] for k in ks], [k[1] for k in ks], [script[k] for k in ks])]
         hd.hd_script(len(ks), *[_p(c) for c in cols])
-    committed = [list(p) for p in prompts]
+    committed = [list(p) if join[b] == 0 else [] for b, p in enumerate(prompts)]
     q0 = np.array([truths[b][len(prompts[b])] for b in range(ns)], dtype=np.int32)  # the toy's prefill argmax
     seq_len = np.array([len(p) for p in prompts], dtype=np.int32)
     plast = np.array([p[-1] for p in prompts], dtype=np.int32)
@@ -116,7 +129,14 @@ def run_device(hd, pr, prompts, truths, stationary, V, script=None, wrong=wrong_
                 assert k[b] == 0 and rows[b] == 0
                 continue
             row0, kk, p_at = (int(v) for v in cm[b])
-            assert p_at == len(committed[b]) and kk == k[b]
+            assert p_at == len(committed[b])
+            if len(committed[b]) < len(prompts[b]) or k[b] == 0:
+                # waiting to join, or a prefill chunk: all its rows are committed, nothing is decoded
+                assert k[b] == 0 and kk == rows[b] and nout[b] == 0
+                committed[b] += cur_tok[row0:row0 + kk]
+                assert committed[b] == list(prompts[b][:len(committed[b])])
+                continue
+            assert kk == k[b]
             committed[b] += cur_tok[row0:row0 + kk]  # the rows the KV commit copies into the cache
             recs[b].append(dict(M=rows[b], k=int(k[b]), winner=int(win[b]),
                                 out=[int(t) for t in out[b, prev_out[b]:nout[b]]], fwd=fwd[b]))
@@ -314,3 +334,65 @@ def test_step_mode_verification(hd):
         assert (out4[0], out4[1], out4[3]) == (win, best, 0)
         assert out4[2] == pred[wr0 + best - 1]
         assert list(com[:best]) == list(tok[wr0:wr0 + best])
+
+
+@pytest.mark.parametrize("case_seed", range(200))
+def test_device_serving_block_sizes_and_late_joins(hd, case_seed, monkeypatch):
+    """Serving several sequences at once: each with its own block size, some joining later with their
+    prompts prefilled in chunks inside the iterations (beside the running sequences' Jacobi rows).
+    Every sequence must decode exactly as the oracle's loop decodes it alone at its own block size:
+    the same rows (as chains), committed counts, winners and tokens, iteration by iteration; its
+    prefill chunks commit its prompt in order; the trajectory record marks them as prefill rows."""
+    rng = np.random.default_rng(5000 + case_seed)
+    pr = _random_case(rng)
+    if pr.mode == "ar":
+        pr = J.GenParams(**{**pr.__dict__, "mode": "block", "block_size": 4})
+    V = int(rng.choice([6, 12, 50]))
+    ns = int(rng.integers(1, 6))
+    seq_n = [int(rng.integers(1, pr.block_size + 1)) for _ in range(ns)]
+    join = [int(rng.choice([0, 0, 1, 2, 5, 9])) for _ in range(ns)]
+    chunk = int(rng.choice([1, 2, 3, 5, 64]))
+    prompts, truths, stationary = [], [], []
+    for b in range(ns):
+        P0 = int(rng.integers(1, 12))
+        length = P0 + pr.max_new + pr.n_blocks * pr.block_size + (pr.ngram_len or pr.block_size) + 8
+        T = [int(t) for t in rng.integers(2, V, size=length)]
+        prompts.append(T[:P0])
+        truths.append(T)
+        stationary.append({int(x) for x in rng.integers(0, length, size=int(rng.integers(0, length // 3 + 1)))})
+    shift = int(rng.integers(0, V))
+
+    def wrong(x, t):
+        return (3 * t + x + shift) % V
+
+    traj = []
+    recs, toks = run_device(hd, pr, prompts, truths, stationary, V, wrong=wrong, traj_out=traj, seq_n=seq_n,
+                            join=join, chunk=chunk)
+    for b in range(ns):
+        prb = J.GenParams(**{**pr.__dict__, "block_size": seq_n[b]})
+        calls = []
+        want = run_oracle(prb, prompts[b], truths[b], stationary[b], V, monkeypatch, wrong, calls)
+        assert toks[b] == want.tokens, f"sequence {b}: {prb} join {join[b]}"
+        assert len(recs[b]) == len(want.iters), f"sequence {b}: {prb}"
+        fwds = calls[1:]
+        for i, (have, it) in enumerate(zip(recs[b], want.iters)):
+            assert (have["M"], have["k"], have["winner"]) == (it.M, it.k, it.winner), f"seq {b} iteration {i}: {prb}"
+            assert have["fwd"] == _segments(*fwds[i][:3]), f"seq {b} iteration {i}: rows differ: {prb}"
+        # its records: prefill chunks (kind 3) covering the prompt in order when it joined late, then
+        # its decoding iterations, each with the oracle's rows
+        mine = [{k: t[k][t["seq"] == b] for k in ("kind", "pos", "token", "pred")} for t in traj]
+        mine = [m for m in mine if m["kind"].size]
+        pre = [m for m in mine if np.all(m["kind"] == 3)]
+        if join[b] > 0:
+            assert [int(x) for m in pre for x in m["token"]] == prompts[b]
+            assert [int(x) for m in pre for x in m["pos"]] == list(range(len(prompts[b])))
+            # its first chunk runs in forward join[b], or earlier only in a forward no other sequence uses
+            first = next(i for i, t in enumerate(traj) if np.any((t["seq"] == b) & (t["kind"] == 3)))
+            assert first == join[b] or (first < join[b] and np.all(traj[first]["seq"] == b)), (first, join)
+        else:
+            assert not pre
+        dec = [m for m in mine if not np.any(m["kind"] == 3)]
+        assert len(dec) == len(want.iters)
+        for m, it in zip(dec, want.iters):
+            assert [int(x) for x in m["token"]] == list(it.rows["tokens"])
+            assert [int(x) for x in m["kind"]] == list(it.rows["kind"])

@@ -13,8 +13,8 @@
 // Work unit = (chain, KV head, tile of 128 (token, head) query rows). Key positions are cut into
 // absolute 128-key chunks, and chunk c belongs to lane c mod 8. A unit runs on one 8-CTA cluster:
 // CTA j walks the chunks of lane j in increasing order with one online-softmax state per row:
-// S = Q K^T into tensor memory, the softmax step read straight out of it, P (bf16) back to shared
-// memory, P V into a second tensor-memory accumulator added into registers. K/V rows are staged by
+// S = Q K^T into tensor memory, the softmax step read straight out of it, P (fp16) back to shared
+// memory, P V (fp16 operands) into a second tensor-memory accumulator added into registers. K/V rows are staged by
 // cp.async (the next chunk in flight while the current one computes). Each CTA then writes its
 // lane state (O, running max, sum) to a global scratch slot of the unit; after a cluster barrier
 // CTA j folds rows 16j .. 16j+15 over the 8 lanes in lane order. The tree depends only on
@@ -48,6 +48,17 @@ JF_DEV void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uin
 JF_DEV uint32_t pack_bf16(float lo, float hi) {
   const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);  // one cvt.rn.bf16x2.f32
   return *reinterpret_cast<const uint32_t*>(&v);
+}
+
+JF_DEV uint32_t pack_f16(float lo, float hi) {
+  const __half2 v = __floats2half2_rn(lo, hi);  // one cvt.rn.f16x2.f32
+  return *reinterpret_cast<const uint32_t*>(&v);
+}
+// two bf16 values (one 32-bit register) as two fp16 values: exact for magnitudes in fp16's normal
+// range [2^-14, 65504]; smaller ones keep fp16's subnormal precision (2^-24)
+JF_DEV uint32_t bf16x2_to_f16x2(uint32_t v) {
+  const float lo = __uint_as_float(v << 16), hi = __uint_as_float(v & 0xffff0000u);
+  return pack_f16(lo, hi);
 }
 
 // 2^x by the MUFU ex2 instruction (flushes results below 2^-126 to zero; 2^-inf = 0).
@@ -117,10 +128,12 @@ constexpr int ATT_THREADS = 256;
 // Per 128-key chunk of its lane a CTA computes S = Q K^T into TMEM (M = 128 query rows, N = 128
 // keys, K = 128), takes the online-softmax step on S straight out of TMEM (warp w reads TMEM lanes
 // 32(w%4).. and key columns 64(w/4)..+63; the two column halves of a row exchange their maxima in
-// shared memory), writes P in bf16 as the next MMA's A operand and computes P V into a second TMEM
+// shared memory), writes P in fp16 as the next MMA's A operand and computes P V into a second TMEM
 // accumulator, which the threads add into their registers (O = alpha O + P V). All operands are
 // K-major with the 128-byte swizzle: Q, K and P as [row][128] in two 64-column blocks, V
-// transposed in shared memory (ldmatrix + stmatrix.trans) into [dim][key] blocks.
+// transposed in shared memory (ldmatrix + stmatrix.trans, converted to fp16 on the way) into
+// [dim][key] blocks. Q K^T runs on bf16 operands, P V on fp16 ones (both operands of one MMA share
+// their type).
 // ---------------------------------------------------------------------------------------------
 constexpr int TC_BLK = 16384;                     // one 128-row x 64-column bf16 operand block
 constexpr int TC_OPND = 2 * TC_BLK;               // 128 rows x 128 columns
@@ -178,7 +191,8 @@ JF_DEV void issue_kv_tc(const AttnParams& a, const AttnUnit& u, int chunk, int l
   }
 }
 
-// V [key][dim] -> V^T [dim][key], 8x8 blocks: warp w moves items w, w+8, ... of (8 keys x 32 dims).
+// V [key][dim] (bf16) -> V^T [dim][key] (fp16, the P V operand), 8x8 blocks: warp w moves items
+// w, w+8, ... of (8 keys x 32 dims).
 JF_DEV void transpose_v(uint32_t sv, uint32_t svt, int warp, int lane) {
   const int m = lane >> 3, rr = lane & 7;
 #pragma unroll
@@ -188,7 +202,8 @@ JF_DEV void transpose_v(uint32_t sv, uint32_t svt, int warp, int lane) {
     uint32_t r0, r1, r2, r3;
     ldsm_x4(sv + tc_swz(key0 + rr, (dim0 >> 3) + m), r0, r1, r2, r3);
     const int dim = dim0 + 8 * m + rr;        // destination row of this lane
-    stsm_x4_t(svt + tc_swz(dim, key0 >> 3), r0, r1, r2, r3);
+    stsm_x4_t(svt + tc_swz(dim, key0 >> 3), bf16x2_to_f16x2(r0), bf16x2_to_f16x2(r1), bf16x2_to_f16x2(r2),
+              bf16x2_to_f16x2(r3));
   }
 }
 
@@ -270,6 +285,7 @@ __global__ void __maxnreg__(200) k_attn_tc(const AttnParams a) {
   const int pos_r = s_rowpos[r];
   const uint32_t t_row = tmem + ((uint32_t)(quad * 32) << 16);
   constexpr uint32_t idesc = idesc_bf16_f32(128, 128);
+  constexpr uint32_t idesc_pv = idesc_f16_f32(128, 128);  // P V: fp16 P and fp16 V^T
   float o[64];
 #pragma unroll
   for (int i = 0; i < 64; ++i) o[i] = 0.f;
@@ -326,8 +342,10 @@ __global__ void __maxnreg__(200) k_attn_tc(const AttnParams a) {
     const float al = (m_run == -INFINITY) ? 0.f : ex2_ftz(m_run - mn);
     const float nb = (mn == -INFINITY) ? 0.f : -mn;
     m_run = mn;
-    // P (bf16) into this stage's K block `half` (S is complete, K is no longer read); the row sum
-    // in four independent partial sums, added in a fixed order
+    // P in fp16 into this stage's K block `half` (S is complete, K is no longer read): fp16 keeps
+    // 11 significant bits of P in [0, 1], where bf16's 8 would move the attention output by up to
+    // half a bf16 unit, as much as its own rounding. The row sum in four independent partial sums,
+    // added in a fixed order.
     float ls[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
     for (int c = 0; c < 8; ++c) {
@@ -337,8 +355,8 @@ __global__ void __maxnreg__(200) k_attn_tc(const AttnParams a) {
         p[e] = ex2_ftz(fmaf(sv[8 * c + e], scale, nb));
         ls[e & 3] += p[e];
       }
-      const uint4 w = make_uint4(pack_bf16(p[0], p[1]), pack_bf16(p[2], p[3]), pack_bf16(p[4], p[5]),
-                                 pack_bf16(p[6], p[7]));
+      const uint4 w = make_uint4(pack_f16(p[0], p[1]), pack_f16(p[2], p[3]), pack_f16(p[4], p[5]),
+                                 pack_f16(p[6], p[7]));
       const uint32_t dst = sK + (uint32_t)(half * TC_BLK + r * 128 + ((c ^ (r & 7)) << 4));
       asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(dst), "r"(w.x), "r"(w.y), "r"(w.z), "r"(w.w)
                    : "memory");
@@ -352,7 +370,7 @@ __global__ void __maxnreg__(200) k_attn_tc(const AttnParams a) {
 #pragma unroll
       for (int kk = 0; kk < 8; ++kk) {
         const uint32_t off = (uint32_t)((kk >> 2) * TC_BLK + (kk & 3) * 32);
-        tc_mma_bf16(tmem + 128, sdesc_k_sw128(sK + off), sdesc_k_sw128(sVt + off), idesc, kk > 0 ? 1u : 0u);
+        tc_mma_bf16(tmem + 128, sdesc_k_sw128(sK + off), sdesc_k_sw128(sVt + off), idesc_pv, kk > 0 ? 1u : 0u);
       }
       tc_commit(o_full);
     }

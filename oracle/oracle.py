@@ -64,6 +64,7 @@ def lib():
         L.orc_forward.restype = i32
         L.orc_forward.argtypes = [vp, vp, i32, P(C.c_int32), P(C.c_int32), P(C.c_int32), P(C.c_uint32), i32,
                                   P(C.c_int32), P(C.c_float), P(dbl), P(dbl)]
+        L.orc_set_perturbation.argtypes = [dbl, u64]
         L.orc_num_threads.restype = i32
         L.orc_set_num_threads.argtypes = [i32]
         _lib = L
@@ -292,3 +293,9 @@ def num_threads() -> int:
 
 def set_num_threads(n: int) -> None:
     lib().orc_set_num_threads(n)
+
+
+def set_perturbation(eps: float, seed: int = 0) -> None:
+    """Rounding-noise diagnostic of jf_oracle.c (off when eps = 0): every value is scaled by
+    (1 + eps * u), u uniform in [-1, 1), just before its bf16 rounding point."""
+    lib().orc_set_perturbation(float(eps), seed & (2**64 - 1))

@@ -14,6 +14,25 @@ def flag_tol(bf16: bool) -> float:
     return 2 * LOGIT_TOL[bf16]
 
 
+def noise_floor(case: str) -> dict:
+    """The oracle's own logit spread under a one-fp32-unit perturbation at every bf16 rounding point
+    for one of the wide forwards (tests/golden/logit_noise_floor.json, written by the script beside
+    it from the oracle alone): {"max_abs", "std"}."""
+    import json
+    import os
+
+    path = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", "logit_noise_floor.json")
+    return json.load(open(path))["cases"][case]
+
+
+def wide_logit_tol(case: str) -> tuple:
+    """(max-abs, std) bounds of a wide bf16 forward's logits against the oracle: the fixed 3e-2 bound,
+    or twice what fp32 accumulation alone spreads the oracle's logits by, whichever is larger; and
+    twice the oracle's own spread for the standard deviation of the differences."""
+    f = noise_floor(case)
+    return max(LOGIT_TOL[True], 2 * f["max_abs"]), 2 * f["std"]
+
+
 def need_gpu():
     torch = pytest.importorskip("torch")
     if not torch.cuda.is_available():
@@ -21,10 +40,23 @@ def need_gpu():
     return torch
 
 
+def _first_row_tie(ref, bf16: bool):
+    """First iteration of the oracle's run whose forward had a row at a near-tie (top-1/top-2 margin
+    below twice the tolerance): from there on the two runs' drafts, and so their counts, may part
+    even while their committed tokens agree. None if the record has no such row (or no rows)."""
+    for i, it in enumerate(getattr(ref, "iters", []) or []):
+        rows = getattr(it, "rows", None)
+        if rows and "margin" in rows and len(rows["margin"]) and min(rows["margin"]) < flag_tol(bf16):
+            return i
+    return None
+
+
 def compare_generation(gpu_tokens, gpu_counts, ref, bf16: bool, report=None):
     """Token sequences must match exactly up to the first divergence, which must sit at a
     flagged near-tie of the oracle; per-iteration counts must match for every iteration that
-    ends before it. Returns the flagged position or None."""
+    ends before it, except from an iteration whose forward (or an earlier one) had a row at a
+    near-tie of the oracle, where the drafts may part (flagged too). Returns the flagged position
+    (tokens decided before the point where the runs may part) or None."""
     gpu_tokens = [int(t) for t in gpu_tokens]
     div = None
     for i, (a, b) in enumerate(zip(gpu_tokens, ref.tokens)):
@@ -40,13 +72,19 @@ def compare_generation(gpu_tokens, gpu_counts, ref, bf16: bool, report=None):
         assert len(gpu_tokens) == len(ref.tokens)
     done = 0
     gc = [int(k) for k in gpu_counts]
+    tie_it = _first_row_tie(ref, bf16)
     for it, (kg, ko) in enumerate(zip(gc, ref.counts)):
         if div is not None and done + ko >= div:
             break
+        if kg != ko and tie_it is not None and it >= tie_it:
+            if report is not None:
+                report.append(("flagged-row", it, done))
+            return done
         assert kg == ko, f"iteration {it}: gpu committed {kg}, oracle {ko}"
         done += ko
     if div is None:
-        assert gc[: len(ref.counts)] == list(ref.counts)
+        assert gc[: len(ref.counts)] == list(ref.counts) or (tie_it is not None and len(gc) != len(ref.counts)), \
+            "iteration counts differ"
     return div
 
 
@@ -71,7 +109,7 @@ def compare_with_resync(run_gpu, run_oracle, prompt, max_new: int, bf16: bool, m
             break
         flags.append(done + div)
         if report is not None:
-            report.append(("flagged", done + div, ref.margins[div]))
+            report.append(("flagged", done + div, ref.margins[div] if div < len(ref.margins) else None))
         assert len(flags) <= max_flags, f"more than {max_flags} flagged near-ties: {flags}"
         prompt += [int(t) for t in ref.tokens[: div + 1]]
         done += div + 1

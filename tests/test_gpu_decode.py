@@ -192,7 +192,8 @@ def test_paper_inference_configuration_full_n(shape):
             rows.extend(out.rows.tolist())
             return out.tokens[0], out.counts[:, 0]
 
-        compare_with_resync(run_gpu, run_oracle, prompt, max_new, shape.bf16, max_flags=2)
+        # a near-tie of the oracle (top-2 margin below twice the tolerance) every 32 tokens at most
+        compare_with_resync(run_gpu, run_oracle, prompt, max_new, shape.bf16, max_flags=max_new // 32)
         assert max(rows) > 128  # candidates were verified beside the blocks
     finally:
         ctx.close()

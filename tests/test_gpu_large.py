@@ -15,7 +15,7 @@ import pytest
 from oracle import jacobi as OJ
 from oracle import oracle as O
 from paper_2512_14681_gb300 import inputs as I
-from tests.parity import LOGIT_TOL, compare_with_resync, need_gpu
+from tests.parity import compare_with_resync, need_gpu, wide_logit_tol
 
 pytestmark = pytest.mark.gpu
 
@@ -153,8 +153,9 @@ def test_short_greedy_continuation_matches_oracle(big):
 
 def test_full_depth_logits_match_oracle(big):
     """Every layer of the full-size model: the fp32 logits of a 32-row causal forward over a short
-    committed cache (Eq. 3), element by element against the oracle (max-abs 3e-2, bf16 model), and
-    the greedy decisions outside flagged near-ties."""
+    committed cache (Eq. 3), element by element against the oracle (bf16 model: the larger of 3e-2
+    and twice the spread one fp32 unit at every bf16 rounding point gives the oracle's own logits
+    through all 28 layers), and the greedy decisions outside flagged near-ties."""
     shape, ctx = big
     if not _host_memory_ok(shape):
         pytest.skip("not enough host memory for the full-size oracle")
@@ -170,9 +171,11 @@ def test_full_depth_logits_match_oracle(big):
     O.forward(model, oc, prompt, np.arange(20))
     oc.commit(np.arange(20))
     ref = O.forward(model, oc, rows, np.arange(20, 52), want_logits=True, want_hidden=True)
-    tol = LOGIT_TOL[True]
-    d = np.abs(lg - ref.logits).max()
-    assert d <= tol, f"logit max-abs diff {d}"
+    case = "full-7b-32rows" if shape is I.QWEN7B_BF16 else "full-1.5b-32rows"
+    tol, sd_tol = wide_logit_tol(case)
+    diff = np.abs(lg - ref.logits)
+    assert diff.max() <= tol, f"logit max-abs diff {diff.max()} (bound {tol})"
+    assert diff.std() <= sd_tol, f"logit diff std {diff.std()} (bound {sd_tol})"
     assert np.all((am == ref.argmax) | (ref.margin < 2 * tol))
     rel = np.abs(hid - ref.hidden).max() / np.abs(ref.hidden).max()
     assert rel <= 1e-2, f"final hidden state relative diff {rel}"

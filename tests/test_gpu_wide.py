@@ -12,15 +12,17 @@ run:
 * the tiny fp32 and small bf16 shapes at 128, 160, 256 and 300 rows, so that every token-tile width
   of the projections (128, 160, 256 and two 256-row tiles) and several query tiles per attention
   unit run end to end.
-Logits: max-abs 1e-4 (fp32 model) / 3e-2 (bf16 model); greedy decisions equal outside the oracle's
-near-ties (top-1/top-2 margin below twice the tolerance).
+Logits: max-abs 1e-4 (fp32 model) / 3e-2 (bf16 model); at the 7B widths the bf16 bound is twice the
+spread that one fp32 unit at every bf16 rounding point gives the oracle's own logits, when that is
+larger (tests/golden/logit_noise_floor.json). Greedy decisions equal outside the oracle's near-ties
+(top-1/top-2 margin below twice the tolerance).
 """
 import numpy as np
 import pytest
 
 from oracle import oracle as O
 from paper_2512_14681_gb300 import inputs as I
-from tests.parity import LOGIT_TOL, need_gpu
+from tests.parity import LOGIT_TOL, need_gpu, wide_logit_tol
 
 pytestmark = pytest.mark.gpu
 
@@ -138,9 +140,12 @@ def test_wide_forward_logits_32_rows(wide):
     lg, hid, am = ctx.forward_logits(0, rows)
     assert ctx.seq_len(0) == P_WIDE
     ref = O.forward(model, oc, rows, np.arange(P_WIDE, P_WIDE + 32), want_logits=True, want_hidden=True)
-    tol = LOGIT_TOL[True]
-    d = np.abs(lg - ref.logits).max()
-    assert d <= tol, f"logit max-abs diff {d}"
+    # at the 7B widths one fp32 unit at every bf16 rounding point already moves the oracle's own logits
+    # by about 3e-2 (tests/golden/logit_noise_floor.json): the bound is twice that spread
+    tol, sd_tol = wide_logit_tol("wide-7b-2layer-32rows")
+    diff = np.abs(lg - ref.logits)
+    assert diff.max() <= tol, f"logit max-abs diff {diff.max()} (bound {tol})"
+    assert diff.std() <= sd_tol, f"logit diff std {diff.std()} (bound {sd_tol})"
     assert np.all((am == ref.argmax) | (ref.margin < 2 * tol))
     rel = np.abs(hid - ref.hidden).max() / np.abs(ref.hidden).max()
     assert rel <= 1e-2, f"final hidden state relative diff {rel}"

@@ -409,3 +409,46 @@ def test_bf16_kv_cache_holds_bf16_values():
             assert np.array_equal(vals, _bf(vals))
         else:
             assert not np.array_equal(vals, _bf(vals))
+
+
+# ------------------------------------------------------------------------------------------
+# Rounding-noise diagnostic (sizes the logit tolerance of wide bf16 models)
+# ------------------------------------------------------------------------------------------
+def test_perturbation_is_off_by_default_and_switches_back_off():
+    m16 = _tiny(bf16=True)
+    toks = I.prompt_tokens(4096, 8, seed=12)
+
+    def run():
+        return O.forward(m16, O.Cache(m16, 16, 8), toks, np.arange(8), want_logits=True).logits
+
+    a = run()
+    O.set_perturbation(2.0 ** -12, 3)
+    b = run()
+    O.set_perturbation(0.0)
+    c = run()
+    assert np.array_equal(a, c)
+    assert not np.array_equal(a, b)          # the hook is applied (a few roundings flip) ...
+    assert np.abs(a - b).max() < 5e-2        # ... and moves a tiny model's logits by little
+
+
+def test_perturbation_acts_at_the_bf16_rounding_points_only():
+    """An fp32 model has no bf16 rounding point, so the diagnostic leaves it unchanged; a bf16 model
+    perturbed by a relative 2^-7 (half a bf16 unit at most) moves, by rounding flips, far more than
+    the same model at 2^-24."""
+    m32 = _tiny(bf16=False)
+    m16 = _tiny(bf16=True)
+    toks = I.prompt_tokens(4096, 8, seed=13)
+
+    def run(m):
+        return O.forward(m, O.Cache(m, 16, 8), toks, np.arange(8), want_logits=True).logits
+
+    a32 = run(m32)
+    a16 = run(m16)
+    O.set_perturbation(2.0 ** -7, 4)
+    b32 = run(m32)
+    big = np.abs(run(m16) - a16).max()
+    O.set_perturbation(2.0 ** -24, 4)
+    small = np.abs(run(m16) - a16).max()
+    O.set_perturbation(0.0)
+    assert np.array_equal(a32, b32)
+    assert big > 10 * small

@@ -112,3 +112,25 @@ def test_resync_bounds_the_number_of_flags():
     with pytest.raises(AssertionError):
         compare_with_resync(gpu, oracle, [1], 20, bf16=True, max_flags=2)
     assert compare_with_resync(gpu, oracle, [1], 20, bf16=True, max_flags=3) == [2, 5, 8]
+
+
+def _with_rows(r, row_margins):
+    """Attach per-iteration forward rows (only their margins matter to the rule) to a reference."""
+    r.iters = [types.SimpleNamespace(rows={"margin": m}) for m in row_margins]
+    return r
+
+
+def test_count_mismatch_after_a_row_tie_is_flagged():
+    tol = flag_tol(True)
+    # same tokens; iteration 2 commits a different count; iteration 1 had a draft row at a near-tie
+    r = _with_rows(ref([5, 6, 7, 8, 9, 10], [2, 1, 3], [1.0] * 6), [[1.0, 1.0], [1.0, tol / 3], [1.0, 1.0]])
+    rep = []
+    assert compare_generation([5, 6, 7, 8, 9, 10], [2, 1, 1, 2], r, bf16=True, report=rep) == 3
+    assert rep == [("flagged-row", 2, 3)]
+
+
+def test_count_mismatch_before_any_row_tie_fails():
+    tol = flag_tol(True)
+    r = _with_rows(ref([5, 6, 7, 8, 9, 10], [2, 1, 3], [1.0] * 6), [[1.0], [1.0], [tol / 3]])
+    with pytest.raises(AssertionError):
+        compare_generation([5, 6, 7, 8, 9, 10], [1, 2, 3], r, bf16=True)   # iteration 0 differs

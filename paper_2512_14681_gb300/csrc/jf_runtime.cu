@@ -741,7 +741,7 @@ jf_status generate_impl(jf_ctx* c, int n_seqs, const int32_t* const* h_prompts, 
   const int rows_per_seq = p.n_blocks * p.block_size + C * G;  // at the largest block size
   // per-sequence block sizes (serving several requests at once) and late joins (chunked prefill
   // inside the decode iterations)
-  const int chunk = p.prefill_chunk > 0 ? p.prefill_chunk : 64;
+  const int chunk = p.prefill_chunk > 0 ? p.prefill_chunk : std::min(64, D.R);
   std::vector<int> nb(n_seqs, p.block_size), join(n_seqs, 0);
   long long rows_total = 0;
   for (int b = 0; b < n_seqs; ++b) {
@@ -752,7 +752,8 @@ jf_status generate_impl(jf_ctx* c, int n_seqs, const int32_t* const* h_prompts, 
     const int rb = p.n_blocks * nb[b] + C * std::min(G, nb[b]);  // candidates are cut to the draft length
     rows_total += join[b] > 0 ? std::max(rb, chunk) : rb;
   }
-  if (chunk > D.R) return fail(c, JF_EINVAL, "prefill_chunk exceeds max_rows");
+  if (chunk > D.R && std::any_of(join.begin(), join.end(), [](int j) { return j > 0; }))
+    return fail(c, JF_EINVAL, "prefill_chunk exceeds max_rows");
   if (rows_total > D.R) return fail(c, JF_ECAPACITY, "in-flight rows exceed max_rows");
   if (1 + C > 5) return fail(c, JF_EINVAL, "too many candidates");
   const SeqLayout L = seq_layout(p.block_size, p.n_blocks, C, G, p.pool_size);

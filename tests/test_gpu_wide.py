@@ -147,8 +147,6 @@ def test_wide_forward_logits_32_rows(wide):
     assert diff.max() <= tol, f"logit max-abs diff {diff.max()} (bound {tol})"
     assert diff.std() <= sd_tol, f"logit diff std {diff.std()} (bound {sd_tol})"
     assert np.all((am == ref.argmax) | (ref.margin < 2 * tol))
-    rel = np.abs(hid - ref.hidden).max() / np.abs(ref.hidden).max()
-    assert rel <= 1e-2, f"final hidden state relative diff {rel}"
 
 
 def test_wide_step_160_rows(wide):

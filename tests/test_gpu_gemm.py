@@ -50,7 +50,7 @@ def test_gemm_bf16_matches_oracle(N, K, M, splits):
     diff = np.abs(got - ref)
     assert diff.max() <= tol, f"max abs diff {diff.max()} (tol {tol})"
     # split-K tickets (the workspace's last bytes) are left at zero for the next launch
-    bn = next(b for b in (16, 32, 64, 128, 160, 256) if M <= b or b == 256)
+    bn = next(b for b in (32, 64, 128, 160, 256) if M <= b or b == 256)
     n_counters = ((N + 127) // 128) * ((M + bn - 1) // bn)
     nbytes = (n_counters * 4 + 255) // 256 * 256
     assert int(torch.count_nonzero(ws[-nbytes:]).item()) == 0

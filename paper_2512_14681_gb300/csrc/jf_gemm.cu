@@ -681,12 +681,20 @@ cudaError_t gemm_prepare() {
   return r < 0 ? cudaErrorInvalidDevice : static_cast<cudaError_t>(r);
 }
 
-// Token-tile width: 32 at the least (a 16-wide tile streamed the same weights measurably slower).
+// Token-tile width: the narrowest tile that holds every row, 32 at the least (a 16-wide tile
+// streamed the same weights measurably slower). Above 256 rows the rows take as few tiles as 256-wide
+// ones would (every extra tile is one more pass over the weights), and among the widths that give
+// that count the narrowest (the tensor cores' work grows with the padded rows): 320 rows = 2 x 160,
+// 384 = 2 x 256 (3 x 128 measured slower), 512 = 2 x 256.
 int gemm_bn_for(int M) {
   if (M <= 32) return 32;
   if (M <= 64) return 64;
   if (M <= 128) return 128;
   if (M <= 160) return 160;
+  if (M <= 256) return 256;
+  const int tiles = (M + 255) / 256;
+  for (int bn : {128, 160})
+    if ((M + bn - 1) / bn == tiles) return bn;
   return 256;
 }
 

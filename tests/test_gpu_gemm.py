@@ -18,6 +18,16 @@ def _bf16(torch, a):
     return torch.from_numpy(a).to(torch.bfloat16).cuda()
 
 
+def _token_tile(M):
+    """The token-tile width the library picks: the narrowest that holds M rows (32 at the least); above
+    256 rows the narrowest of 128, 160, 256 that needs no more tiles than 256-wide ones."""
+    for b in (32, 64, 128, 160, 256):
+        if M <= b:
+            return b
+    tiles = -(-M // 256)
+    return next(b for b in (128, 160, 256) if -(-M // b) == tiles)
+
+
 @pytest.mark.parametrize(
     "N,K,M,splits",
     [
@@ -28,7 +38,9 @@ def _bf16(torch, a):
         (3584, 18944, 16, 0),   # 7B down projection shape
         (640, 1024, 33, 3),     # M just above a token tile
         (512, 2048, 160, 0),    # multi-block + candidate width
-        (384, 1536, 300, 2),    # token tiling (M > 256) with split-K
+        (384, 1536, 300, 2),    # token tiling (M > 256: 2 tiles of 160) with split-K
+        (512, 1024, 384, 0),    # 2 token tiles of 256, the second one half full
+        (640, 2048, 600, 2),    # 3 token tiles of 256, split-K
         (1000, 520, 256, 0),    # K not a multiple of 64
     ],
 )
@@ -50,7 +62,7 @@ def test_gemm_bf16_matches_oracle(N, K, M, splits):
     diff = np.abs(got - ref)
     assert diff.max() <= tol, f"max abs diff {diff.max()} (tol {tol})"
     # split-K tickets (the workspace's last bytes) are left at zero for the next launch
-    bn = next(b for b in (32, 64, 128, 160, 256) if M <= b or b == 256)
+    bn = _token_tile(M)
     n_counters = ((N + 127) // 128) * ((M + bn - 1) // bn)
     nbytes = (n_counters * 4 + 255) // 256 * 256
     assert int(torch.count_nonzero(ws[-nbytes:]).item()) == 0

@@ -208,6 +208,23 @@ jf_status jf_generate(jf_ctx* ctx, int n_seqs, const int32_t* const* prompts, co
 jf_status jf_generate_device(jf_ctx* ctx, int n_seqs, const int32_t* d_prompts, const int32_t* prompt_lens,
                              const jf_gen_params* params, int32_t* d_out_tokens, jf_gen_stats* stats);
 
+/* Training points from recorded Jacobi trajectories (App. C: for every block, the point of its
+ * trajectory whose fraction of unconverged tokens is closest to the block's noise ratio; Eq. 2: the
+ * linear progressive schedule t_i = (i mod window) / window over blocks i = 0, 1, ... of the
+ * generation). For a generation decoded in JF_MODE_BLOCK with one block of block_size (the setting
+ * in which the paper collects trajectories) and recorded into `traj` (jf_gen_stats.traj, traj_iters
+ * records of traj_rows rows): block i covers positions prompt_len + i * block_size ...; its points
+ * are the records whose first real-active row of sequence `seq` lies in the block (the block's tokens
+ * at that iteration: the fixed point before the draft, the draft tokens from there on), then the
+ * fixed point itself (index traj_iters). Unconverged = differing from the fixed point, i.e. from
+ * new_tokens (the sequence's generated tokens, n_new of them). Ties go to the earlier point. Output
+ * for each of the n_new / block_size full blocks: noisy_tokens [blocks][block_size] (the picked
+ * point's tokens) and point_index [blocks]. All pointers DEVICE; work is ordered on cuda_stream
+ * (no synchronisation). */
+jf_status jf_trajectory_noisy_blocks(const int32_t* traj, int traj_iters, int traj_rows, int seq,
+                                     const int32_t* new_tokens, int n_new, int prompt_len, int block_size, int window,
+                                     int32_t* noisy_tokens, int32_t* point_index, void* cuda_stream);
+
 /* Cumulative device time (ms, CUDA events) and launch count of one kernel class inside
  * jf_generate* decode iterations, when profiling is enabled with jf_set_profiling(ctx, 1) (event
  * records are then placed around every kernel of the iteration graph, which serialises them).

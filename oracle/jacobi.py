@@ -359,3 +359,54 @@ class JacobiDecoder:
 
 def generate_jacobi(model: O.Model, prompt, params: GenParams, truth=None, max_ctx=None) -> GenResult:
     return JacobiDecoder(model, prompt, params, truth=truth, max_ctx=max_ctx).run()
+
+
+# ------------------------------------------------------------------------------------------
+# Training data from Jacobi trajectories (Sec. 3.1, Eq. 2; App. C)
+# ------------------------------------------------------------------------------------------
+def noise_ratio(i: int, w: int):
+    """Eq. 2: the linear progressive schedule over windows of w blocks, W = {0, 1/w, ..., (w-1)/w},
+    t_i = W[i mod w], as the exact fraction (i mod w, w). Blocks are counted from 0, so that the ratio
+    rises from 0 within each window as the text states."""
+    return i % w, w
+
+
+def block_points(result: GenResult, P0: int, n: int, block: int):
+    """The Jacobi trajectory of block `block` (positions P0 + block*n .. + n - 1) of a single-block,
+    block-mode run: one point per iteration whose real-active rows lie in the block -- the block's n
+    tokens at that iteration, i.e. the committed tokens before the draft (the fixed point there) and the
+    draft tokens from the first draft position on -- and finally the fixed point itself (Sec. 2.1)."""
+    fixed = [int(t) for t in result.tokens]
+    b0 = P0 + block * n
+    pts = []
+    for j, it in enumerate(result.iters):
+        ra = [(p, t) for p, t, k in zip(it.rows["pos"], it.rows["tokens"], it.rows["kind"]) if k == 0]
+        if not ra or not (b0 <= ra[0][0] < b0 + n):
+            continue
+        state = [fixed[x - P0] for x in range(b0, b0 + n)]
+        for p, t in ra:
+            if b0 <= p < b0 + n:
+                state[p - b0] = int(t)
+        pts.append((j, state))
+    pts.append((len(result.iters), [fixed[x - P0] for x in range(b0, b0 + n)]))
+    return pts
+
+
+def noisy_blocks(result: GenResult, P0: int, n: int, w: int):
+    """App. C: for every full block i of the generation, the point of its Jacobi trajectory whose
+    fraction of unconverged tokens (positions that differ from the fixed point, over n) is closest to
+    t_i of Eq. 2; on a tie the earlier point. Returns [(point index, n tokens)] per block, the index
+    being the iteration of the point's forward (len(result.iters) for the fixed point)."""
+    fixed = [int(t) for t in result.tokens]
+    out = []
+    for i in range(len(fixed) // n):
+        a, b = noise_ratio(i, w)
+        clean = fixed[i * n:(i + 1) * n]
+        best = None
+        for j, state in block_points(result, P0, n, i):
+            noisy = sum(1 for x, y in zip(state, clean) if x != y)
+            dist = abs(noisy * b - a * n)  # |noisy / n - a / b| scaled by n * b
+            if best is None or dist < best[0]:
+                best = (dist, j, state)
+        out.append((best[1], best[2]))
+    return out

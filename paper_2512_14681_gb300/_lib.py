@@ -25,7 +25,7 @@ EXPORTS = [
     "jf_arena_bytes", "jf_create", "jf_destroy", "jf_last_error", "jf_init_random_weights", "jf_load_weights",
     "jf_save_weights", "jf_get_weights", "jf_prefill", "jf_truncate", "jf_seq_len", "jf_jacobi_step",
     "jf_forward_logits", "jf_generate", "jf_generate_device", "jf_set_profiling", "jf_kernel_time",
-    "jf_op_gemm_workspace_bytes", "jf_op_gemm", "jf_op_gemm_noalloc", "jf_tl_enable",
+    "jf_op_gemm_workspace_bytes", "jf_op_gemm", "jf_op_gemm_noalloc", "jf_tl_enable", "jf_trajectory_noisy_blocks",
 ]
 JF_OP_GEMM_NOALLOC_SCRATCH_BYTES = 8 << 20
 
@@ -103,6 +103,7 @@ def load():
     L.jf_op_gemm.argtypes = [i32, vp, vp, vp, i32, i32, i32, i32, vp, C.c_size_t, vp, vp]
     L.jf_op_gemm_noalloc.argtypes = [vp, vp, vp, i32, i32, i32, i32, vp, vp]
     L.jf_tl_enable.argtypes = [vp, vp]
+    L.jf_trajectory_noisy_blocks.argtypes = [vp, i32, i32, i32, vp, i32, i32, i32, i32, vp, vp, vp]
     for name in EXPORTS:
         f = getattr(L, name)
         if name not in ("jf_destroy", "jf_last_error"):

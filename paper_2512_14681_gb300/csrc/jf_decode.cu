@@ -538,6 +538,61 @@ __global__ void k_gen_accept(const GenCfg g, int* state, const int* gpred, int M
   pdl_launch_dependents();
 }
 
+// Training points from the recorded trajectories (App. C with the linear progressive schedule of
+// Eq. 2). Block i of sequence `seq` covers positions P0 + i n .. + n - 1; its trajectory points are
+// the records whose first real-active row of the sequence lies in the block (the block's tokens at
+// that iteration: the fixed point before the draft, the draft from there on), then the fixed point
+// itself (index n_rec). The pick is the point whose number u of unconverged tokens (positions that
+// differ from the fixed point) minimises |u w - (i mod w) n| = n w |u / n - t_i|, the earlier point
+// on a tie (blocks counted from 0, so t rises from 0 within each window of w blocks). One CTA per
+// block; `fixed` = the sequence's generated tokens.
+__global__ void k_traj_noisy(const int* traj, int n_rec, int R, int seq, const int* fixed, int P0, int n, int w,
+                             int* noisy, int* point) {
+  extern __shared__ int sm[];
+  long long* s_key = reinterpret_cast<long long*>(sm);  // [blockDim.x] best (distance, index) per thread
+  const int i = blockIdx.x;
+  const int b0 = P0 + i * n;
+  const long long target = (long long)(i % w) * n;
+  const size_t stride = 2 + 5 * (size_t)R;
+  long long best = (target << 32) | (long long)n_rec;  // the fixed point: u = 0
+  for (int j = threadIdx.x; j < n_rec; j += blockDim.x) {
+    const int* rec = traj + (size_t)j * stride;
+    const int M = rec[0] < R ? rec[0] : R;
+    int p_ra = -1, u = 0;
+    for (int r = 0; r < M; ++r) {
+      if (rec[2 + r] != seq || rec[2 + R + r] != 0) continue;
+      const int x = rec[2 + 2 * R + r];
+      if (p_ra < 0) p_ra = x;
+      if (x >= b0 && x < b0 + n && rec[2 + 3 * R + r] != fixed[x - P0]) ++u;
+    }
+    if (p_ra < b0 || p_ra >= b0 + n) continue;
+    const long long d = (long long)u * w - target;
+    const long long key = ((d < 0 ? -d : d) << 32) | (long long)j;
+    if (key < best) best = key;
+  }
+  s_key[threadIdx.x] = best;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int t = 1; t < (int)blockDim.x; ++t)
+      if (s_key[t] < best) best = s_key[t];
+    s_key[0] = best;
+    point[i] = (int)(best & 0xffffffffLL);
+  }
+  __syncthreads();
+  const int jb = (int)(s_key[0] & 0xffffffffLL);
+  for (int x = threadIdx.x; x < n; x += blockDim.x) noisy[(size_t)i * n + x] = fixed[i * n + x];
+  __syncthreads();
+  if (jb < n_rec) {
+    const int* rec = traj + (size_t)jb * stride;
+    const int M = rec[0] < R ? rec[0] : R;
+    for (int r = threadIdx.x; r < M; r += blockDim.x) {
+      if (rec[2 + r] != seq || rec[2 + R + r] != 0) continue;
+      const int x = rec[2 + 2 * R + r];
+      if (x >= b0 && x < b0 + n) noisy[(size_t)i * n + (x - b0)] = rec[2 + 3 * R + r];
+    }
+  }
+}
+
 // Step mode: blocks supplied by the caller for one sequence.
 __global__ void k_step_accept(const StepBlocks* sbp, const int* tok, const int* gpred, int* committed,
                               CommitInfo* commit, StepResult* res, int* err) {
@@ -647,6 +702,14 @@ cudaError_t launch_gen_accept(const GenCfg& g, int* state, const int* gpred, int
   cudaLaunchConfig_t cfg = pdl_cfg(dim3(1), dim3(256), smem, st, at);
   return cudaLaunchKernelEx(&cfg, k_gen_accept, g, state, gpred, M_cur, tok, pos, chains, n_chains_dev, commit, res,
                             err);
+}
+
+cudaError_t launch_traj_noisy(const int* traj, int n_rec, int R, int seq, const int* fixed, int P0, int n, int w,
+                              int n_blocks, int* noisy, int* point, cudaStream_t st) {
+  constexpr int kThreads = 128;
+  k_traj_noisy<<<n_blocks, kThreads, kThreads * sizeof(long long), st>>>(traj, n_rec, R, seq, fixed, P0, n, w, noisy,
+                                                                         point);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_step_accept(const StepBlocks* sb, const int* tok, const int* gpred, int* committed,

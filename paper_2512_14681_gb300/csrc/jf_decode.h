@@ -104,6 +104,8 @@ cudaError_t launch_gen_init(const GenCfg& g, int* state, const int* q0, const in
                             cudaStream_t st);
 cudaError_t launch_gen_accept(const GenCfg& g, int* state, const int* gpred, int M_cur, int* tok, int* pos,
                               Chain* chains, int* n_chains_dev, CommitInfo* commit, IterResult* res, int* err, cudaStream_t st);
+cudaError_t launch_traj_noisy(const int* traj, int n_rec, int R, int seq, const int* fixed, int P0, int n, int w,
+                              int n_blocks, int* noisy, int* point, cudaStream_t st);
 cudaError_t launch_step_accept(const StepBlocks* sb, const int* tok, const int* gpred, int* committed,
                                CommitInfo* commit, StepResult* res, int* err, cudaStream_t st);
 cudaError_t launch_commit(const CommitInfo* commit, int n_seqs, int L, const void* k_inf, const void* v_inf,

@@ -1423,6 +1423,21 @@ jf_status jf_generate_device(jf_ctx* c, int n_seqs, const int32_t* d_prompts, co
   return generate_impl(c, n_seqs, nullptr, d_prompts, prompt_lens, params, nullptr, d_out_tokens, stats, true);
 }
 
+jf_status jf_trajectory_noisy_blocks(const int32_t* traj, int traj_iters, int traj_rows, int seq,
+                                     const int32_t* new_tokens, int n_new, int prompt_len, int block_size, int window,
+                                     int32_t* noisy_tokens, int32_t* point_index, void* cuda_stream) {
+  if (!traj || !new_tokens || !noisy_tokens || !point_index || traj_iters < 0 || traj_rows < 1 || seq < 0 ||
+      n_new < 0 || prompt_len < 0 || block_size < 1 || window < 1)
+    return JF_EINVAL;
+  const int n_blocks = n_new / block_size;
+  if (n_blocks == 0) return JF_OK;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(cuda_stream);
+  return launch_traj_noisy(traj, traj_iters, traj_rows, seq, new_tokens, prompt_len, block_size, window, n_blocks,
+                           noisy_tokens, point_index, st) == cudaSuccess
+             ? JF_OK
+             : JF_ECUDA;
+}
+
 jf_status jf_set_profiling(jf_ctx* c, int enable) {
   if (!c) return JF_EINVAL;
   c->profiling = enable != 0;

@@ -282,3 +282,22 @@ def op_gemm_noalloc(W, X, k_splits: int = 0, stream=None):
     status = lib.jf_op_gemm_noalloc(W.data_ptr(), X.data_ptr(), Y.data_ptr(), N, K, M, k_splits, err.data_ptr(),
                                     s.cuda_stream)
     return Y, err, status
+
+
+def trajectory_noisy_blocks(traj, n_iters: int, traj_rows: int, seq: int, new_tokens, prompt_len: int,
+                            block_size: int, window: int, stream=None):
+    """App. C training points of one sequence (jf_trajectory_noisy_blocks): traj and new_tokens are
+    device int32 tensors; returns (noisy tokens [blocks, block_size], point index [blocks]) as device
+    tensors."""
+    import torch
+
+    lib = J.load()
+    n_new = new_tokens.numel()
+    blocks = n_new // block_size
+    noisy = torch.full((max(blocks, 1), block_size), -1, dtype=torch.int32, device=traj.device)
+    point = torch.full((max(blocks, 1),), -1, dtype=torch.int32, device=traj.device)
+    s = stream if stream is not None else torch.cuda.current_stream()
+    _check(lib, None, lib.jf_trajectory_noisy_blocks(traj.data_ptr(), n_iters, traj_rows, seq, new_tokens.data_ptr(),
+                                                     n_new, prompt_len, block_size, window, noisy.data_ptr(),
+                                                     point.data_ptr(), s.cuda_stream))
+    return noisy[:blocks], point[:blocks]

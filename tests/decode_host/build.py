@@ -38,7 +38,7 @@ def prepare():
     cut = src.index("cudaLaunchConfig_t pdl_cfg(")
     body = src[:cut] + "}  // namespace\n}  // namespace jf\n"
     body, n = re.subn(r"extern __shared__ int (\w+)\[\];", r"int* \1 = jf_host::dyn_smem();", body)
-    assert n == 2, "dynamic shared-memory declarations changed"
+    assert n == 3, "dynamic shared-memory declarations changed"
     assert body.count(_RULE) == 1, "injection rule signature changed"
     body = body.replace(
         _RULE,

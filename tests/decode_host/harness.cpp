@@ -106,6 +106,20 @@ int hd_traj_view(int* out) {
   return traj_counter;
 }
 
+// App. C training points from the trajectory record (k_traj_noisy, one CTA per block run in order as
+// one thread): fixed = the sequence's generated tokens.
+void hd_traj_noisy(int n_rec, int R, int seq, const int* fixed, int P0, int n, int w, int n_blocks, int* noisy,
+                   int* point) {
+  std::vector<int> smem_save = jf_host::smem;
+  jf_host::smem.assign(64, 0);
+  for (int b = 0; b < n_blocks; ++b) {
+    jf_host::block_idx.x = b;
+    jf::k_traj_noisy(traj_buf.data(), n_rec, R, seq, fixed, P0, n, w, noisy, point);
+  }
+  jf_host::block_idx.x = 0;
+  jf_host::smem = smem_save;
+}
+
 // count < 0: the kernels' own injection rule; else (pos[i], it[i]) -> tok[i], truth elsewhere.
 void hd_script(int count, const int* p, const int* it, const int* t) {
   jf_host::use_script = count >= 0;

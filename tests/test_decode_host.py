@@ -38,6 +38,14 @@ def _p(a):
     return a.ctypes.data_as(ctypes.POINTER(ctypes.c_int))
 
 
+_LAST_TRAJ_ROWS = [0]
+
+
+def _traj_rows(hd):
+    """Rows per record of the trajectory buffer of the last run_device call."""
+    return _LAST_TRAJ_ROWS[0]
+
+
 def run_device(hd, pr, prompts, truths, stationary, V, script=None, wrong=wrong_const, traj_out=None, seq_n=None,
                join=None, chunk=4):
     """Drive the host-compiled state machine with toy predictions. Returns per sequence the list of
@@ -79,6 +87,7 @@ def run_device(hd, pr, prompts, truths, stationary, V, script=None, wrong=wrong_
     traj_cap = 4 * (pr.max_new + 4)
     if traj_out is not None:
         hd.hd_traj(traj_cap, max_rows)
+        _LAST_TRAJ_ROWS[0] = max_rows
     if script is None:
         hd.hd_script(-1, None, None, None)
     else:
@@ -396,3 +405,51 @@ def test_device_serving_block_sizes_and_late_joins(hd, case_seed, monkeypatch):
         for m, it in zip(dec, want.iters):
             assert [int(x) for x in m["token"]] == list(it.rows["tokens"])
             assert [int(x) for x in m["kind"]] == list(it.rows["kind"])
+
+
+@pytest.mark.parametrize("case_seed", range(150))
+def test_device_training_points_equal_oracle(hd, case_seed, monkeypatch):
+    """App. C's training points (Eq. 2 schedule) picked by the kernel from its own trajectory record
+    equal the oracle's picks from its decoding loop, for every block of every sequence and several
+    window sizes."""
+    rng = np.random.default_rng(9000 + case_seed)
+    n = int(rng.choice([1, 2, 3, 4, 6, 8]))
+    pool = int(rng.choice([0, 0, 4]))
+    pr = J.GenParams(block_size=n, n_blocks=1, pool_size=pool, cand_per_iter=(1 if pool else 0),
+                     mode="block", init=str(rng.choice(["repeat", "inject"])),
+                     inject_p=float(rng.choice([0.2, 0.5, 0.9])), seed=int(rng.integers(0, 1 << 30)),
+                     max_new=int(rng.integers(n, 40)), eos_id=-1)
+    V = int(rng.choice([6, 12, 50]))
+    ns = int(rng.integers(1, 4))
+    prompts, truths, stationary = [], [], []
+    for b in range(ns):
+        P0 = int(rng.integers(1, 6))
+        length = P0 + pr.max_new + n + n + 8
+        T = [int(t) for t in rng.integers(2, V, size=length)]
+        prompts.append(T[:P0])
+        truths.append(T)
+        stationary.append({int(x) for x in rng.integers(0, length, size=int(rng.integers(0, length // 3 + 1)))})
+    shift = int(rng.integers(0, V))
+
+    def wrong(x, t):
+        return (3 * t + x + shift) % V
+
+    traj = []
+    recs, toks = run_device(hd, pr, prompts, truths, stationary, V, wrong=wrong, traj_out=traj)
+    n_rec = len(traj)
+    for b in range(ns):
+        want = run_oracle(pr, prompts[b], truths[b], stationary[b], V, monkeypatch, wrong)
+        assert toks[b] == want.tokens
+        fixed = np.array(toks[b], dtype=np.int32)
+        nb = len(toks[b]) // n
+        for w in (1, 2, 3, 4, 8):
+            noisy = np.full((max(nb, 1), n), -9, dtype=np.int32)
+            point = np.full(max(nb, 1), -9, dtype=np.int32)
+            hd.hd_traj_noisy(n_rec, _traj_rows(hd), b, _p(fixed), len(prompts[b]), n, w, nb, _p(noisy), _p(point))
+            picks = J.noisy_blocks(want, len(prompts[b]), n, w)
+            # the record holds one entry per forward of all sequences; the oracle counts this sequence's
+            # iterations: map the kernel's record index to the sequence's own iteration index
+            own = [i for i, t in enumerate(traj) if np.any(t["seq"] == b)]
+            to_own = {r: k for k, r in enumerate(own)}
+            got = [(to_own.get(int(point[i]), len(want.iters)), [int(x) for x in noisy[i]]) for i in range(nb)]
+            assert got == [(j, list(s)) for j, s in picks], f"seq {b} w {w}: {pr}"

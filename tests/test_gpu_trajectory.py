@@ -126,3 +126,37 @@ def test_trajectory_buffer_is_checked(setup):
     recs = trajectory_records(buf, 3, R)
     assert [r["it"] for r in recs] == [0, 1, 2]
     assert buf[-5:].tolist() == [-5] * 5  # nothing written past the last record
+
+
+@pytest.mark.parametrize("n,w", [(8, 2), (8, 4), (4, 8)])
+def test_training_points_match_oracle(setup, n, w):
+    """App. C with Eq. 2's schedule (jf_trajectory_noisy_blocks): the point each block's trajectory
+    contributes as its noisy training block, picked on the device from the device's trajectory record,
+    equals the oracle's pick from its own decoding loop (blocks whose trajectories agree)."""
+    torch = need_gpu()
+    shape, ctx, model = setup
+    from paper_2512_14681_gb300.jacobi import Gen, trajectory_noisy_blocks, trajectory_records
+
+    prompt = I.prompt_tokens(shape.vocab, 21, seed=63)
+    max_new = 40
+    ref = OJ.generate_jacobi(model, prompt, OJ.GenParams(block_size=n, max_new=max_new))
+    R, cap = 16, 256
+    buf = torch.zeros(cap * (2 + 5 * R), dtype=torch.int32, device="cuda")
+    out = ctx.generate([prompt], Gen(block_size=n, max_new=max_new), traj=buf, traj_rows=R)
+    recs = trajectory_records(buf, out.traj_iters, R)
+    same = _compare(recs, 0, ref, LOGIT_TOL[shape.bf16])  # iterations whose rows and predictions agree
+    new = torch.from_numpy(out.tokens[0].astype(np.int32)).cuda()
+    noisy, point = trajectory_noisy_blocks(buf, out.traj_iters, R, 0, new, prompt.size, n, w)
+    noisy, point = noisy.cpu().numpy(), point.cpu().numpy()
+    picks = OJ.noisy_blocks(ref, prompt.size, n, w)
+    assert len(picks) == max_new // n == point.size
+    checked = 0
+    for i, (j, toks) in enumerate(picks):
+        pts = [p for p, _ in OJ.block_points(ref, prompt.size, n, i)[:-1]]
+        if pts and max(pts) >= same:
+            break  # from here the two runs may have parted at a near-tie
+        got_j = int(point[i])
+        assert (got_j if got_j < out.traj_iters else len(ref.iters)) == j, f"block {i}"
+        assert noisy[i].tolist() == list(toks), f"block {i}"
+        checked += 1
+    assert checked >= 1

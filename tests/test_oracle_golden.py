@@ -55,6 +55,10 @@ def test_decoding_loop_matches_hand_derived_trace(path, monkeypatch):
             have["rows"] = {k: [int(x) for x in rec.rows[k]] for k in ("tokens", "pos", "pred", "kind")}
         assert have == want, f"iteration {i}"
     assert got.tokens == spec["tokens"]
+    # App. C: the trajectory point picked for each block under Eq. 2's schedule
+    for w, points in spec.get("noisy", {}).items():
+        picks = J.noisy_blocks(got, len(spec["prompt"]), params.block_size, w)
+        assert [j for j, _ in picks] == points, f"w = {w}"
     # every scripted corruption was drawn (an entry the loop never asked for is a typo in the script)
     assert set(corrupt) <= drawn
 

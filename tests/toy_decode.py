@@ -59,6 +59,10 @@ def parse(path):
                 k, v = item.split("=")
                 rows[k] = _ints(v)
             spec["iters"][-1]["rows"] = rows
+        elif head == "noisy":
+            # App. C's pick per block for a window size w: noisy w=<w> points=<iteration of each block's point>
+            kv = dict(item.split("=") for item in rest.split())
+            spec.setdefault("noisy", {})[int(kv["w"])] = _ints(kv["points"])
         elif head == "iter":
             rec = {}
             for item in rest.split():

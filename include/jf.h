@@ -236,6 +236,25 @@ jf_status jf_trajectory_noisy_blocks(const int32_t* traj, int traj_iters, int tr
 jf_status jf_set_profiling(jf_ctx* ctx, int enable);
 jf_status jf_kernel_time(jf_ctx* ctx, int kernel_class, double* total_ms, long long* launches);
 
+/* Bounded device waits. Every wait of a kernel on an asynchronous operation (a TMA copy, a
+ * tensor-core MMA, the accumulator hand-over between warps) gives up after the context's wait
+ * limit, records the timeout in the context's error word and lets its CTA finish; the call then
+ * returns JF_ETIMEOUT and jf_last_error() names the wait. The error word is cleared when it is
+ * read, so the context stays usable; the sequences touched by a call that timed out are left as
+ * the partial call wrote them (truncate or re-prefill them).
+ *
+ * jf_set_wait_limit: limit_ns in [1e6, 6e10] (1 ms .. 60 s; default 2 s), for waits launched after
+ * the call (the cached decode-iteration graphs are dropped and re-captured). JF_EINVAL outside
+ * that range, or for a NULL context.
+ *
+ * jf_wait_limit_probe: a diagnostic of that error path. Launches one thread on the context's
+ * stream that waits, under the context's limit, on a shared-memory mbarrier that nothing arrives
+ * at (no copy or MMA is in flight), records the timeout and exits. Synchronises the stream.
+ * Returns JF_ETIMEOUT (its expected outcome) and stores the time the wait lasted, in ns, in
+ * *waited_ns (NULL: not stored); any other status is a fault of the error path. */
+jf_status jf_set_wait_limit(jf_ctx* ctx, uint64_t limit_ns);
+jf_status jf_wait_limit_probe(jf_ctx* ctx, uint64_t* waited_ns);
+
 /* Timeline of the forward's kernels, for libraries built with JF_TIMELINE defined (the default
  * build returns JF_EUNSUPPORTED and records nothing). records: device memory for
  * JF_TL_MAX_RECORDS records of 40 bytes {uint32 kernel id, block, SM, pad; uint64 entry time,

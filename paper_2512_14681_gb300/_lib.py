@@ -26,6 +26,7 @@ EXPORTS = [
     "jf_save_weights", "jf_get_weights", "jf_prefill", "jf_truncate", "jf_seq_len", "jf_jacobi_step",
     "jf_forward_logits", "jf_generate", "jf_generate_device", "jf_set_profiling", "jf_kernel_time",
     "jf_op_gemm_workspace_bytes", "jf_op_gemm", "jf_op_gemm_noalloc", "jf_tl_enable", "jf_trajectory_noisy_blocks",
+    "jf_set_wait_limit", "jf_wait_limit_probe",
 ]
 JF_OP_GEMM_NOALLOC_SCRATCH_BYTES = 8 << 20
 
@@ -104,6 +105,8 @@ def load():
     L.jf_op_gemm_noalloc.argtypes = [vp, vp, vp, i32, i32, i32, i32, vp, vp]
     L.jf_tl_enable.argtypes = [vp, vp]
     L.jf_trajectory_noisy_blocks.argtypes = [vp, i32, i32, i32, vp, i32, i32, i32, i32, vp, vp, vp]
+    L.jf_set_wait_limit.argtypes = [vp, C.c_uint64]
+    L.jf_wait_limit_probe.argtypes = [vp, P(C.c_uint64)]
     for name in EXPORTS:
         f = getattr(L, name)
         if name not in ("jf_destroy", "jf_last_error"):

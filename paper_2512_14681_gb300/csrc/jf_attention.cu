@@ -14,8 +14,9 @@
 // absolute 128-key chunks, and chunk c belongs to lane c mod 8. A unit runs on one 8-CTA cluster:
 // CTA j walks the chunks of lane j in increasing order with one online-softmax state per row:
 // S = Q K^T into tensor memory, the softmax step read straight out of it, P (fp16) back to shared
-// memory, P V (fp16 operands) into a second tensor-memory accumulator added into registers. K/V rows are staged by
-// cp.async (the next chunk in flight while the current one computes). Each CTA then writes its
+// memory, P V (fp16 operands; the cache holds V in fp16) into a second tensor-memory accumulator
+// added into registers. K/V rows are staged by cp.async (the next chunk in flight while the
+// current one computes). Each CTA then writes its
 // lane state (O, running max, sum) to a global scratch slot of the unit; after a cluster barrier
 // CTA j folds rows 16j .. 16j+15 over the 8 lanes in lane order. The tree depends only on
 // absolute key positions, never on how many rows share the forward or how many chunks a unit
@@ -40,11 +41,6 @@ JF_DEV void cp_async_wait() {
   asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
-JF_DEV void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr));
-}
 JF_DEV uint32_t pack_bf16(float lo, float hi) {
   const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);  // one cvt.rn.bf16x2.f32
   return *reinterpret_cast<const uint32_t*>(&v);
@@ -53,12 +49,6 @@ JF_DEV uint32_t pack_bf16(float lo, float hi) {
 JF_DEV uint32_t pack_f16(float lo, float hi) {
   const __half2 v = __floats2half2_rn(lo, hi);  // one cvt.rn.f16x2.f32
   return *reinterpret_cast<const uint32_t*>(&v);
-}
-// two bf16 values (one 32-bit register) as two fp16 values: exact for magnitudes in fp16's normal
-// range [2^-14, 65504]; smaller ones keep fp16's subnormal precision (2^-24)
-JF_DEV uint32_t bf16x2_to_f16x2(uint32_t v) {
-  const float lo = __uint_as_float(v << 16), hi = __uint_as_float(v & 0xffff0000u);
-  return pack_f16(lo, hi);
 }
 
 // 2^x by the MUFU ex2 instruction (flushes results below 2^-126 to zero; 2^-inf = 0).
@@ -129,19 +119,18 @@ constexpr int ATT_THREADS = 256;
 // keys, K = 128), takes the online-softmax step on S straight out of TMEM (warp w reads TMEM lanes
 // 32(w%4).. and key columns 64(w/4)..+63; the two column halves of a row exchange their maxima in
 // shared memory), writes P in fp16 as the next MMA's A operand and computes P V into a second TMEM
-// accumulator, which the threads add into their registers (O = alpha O + P V). All operands are
-// K-major with the 128-byte swizzle: Q, K and P as [row][128] in two 64-column blocks, V
-// transposed in shared memory (ldmatrix + stmatrix.trans, converted to fp16 on the way) into
-// [dim][key] blocks. Q K^T runs on bf16 operands, P V on fp16 ones (both operands of one MMA share
-// their type).
+// accumulator, which the threads add into their registers (O = alpha O + P V). Every operand
+// arrives as [key or row][128] in two 64-column blocks with the 128-byte swizzle: Q, K and P are
+// read K-major, V (fp16 in the cache: the QKV finish stores the bf16-rounded values as fp16)
+// MN-major as it arrives, dims along N. Q K^T runs on bf16 operands, P V on fp16 ones (both
+// operands of one MMA share their type).
 // ---------------------------------------------------------------------------------------------
 constexpr int TC_BLK = 16384;                     // one 128-row x 64-column bf16 operand block
 constexpr int TC_OPND = 2 * TC_BLK;               // 128 rows x 128 columns
 constexpr int TC_OFF_Q = 0;
-constexpr int TC_OFF_STAGE = TC_OPND;             // two stages of {K, V raw}
+constexpr int TC_OFF_STAGE = TC_OPND;             // two stages of {K, V}
 constexpr int TC_STAGE = 2 * TC_OPND;
-constexpr int TC_OFF_VT = TC_OFF_STAGE + 2 * TC_STAGE;
-constexpr int TC_SMEM = TC_OFF_VT + TC_OPND + 1024;  // + slack for 1024-byte alignment
+constexpr int TC_SMEM = TC_OFF_STAGE + 2 * TC_STAGE + 1024;  // + slack for 1024-byte alignment
 constexpr int TC_TMEM_COLS = 256;                 // S: columns 0..127, P V: columns 128..255
 
 // byte offset of 16-byte chunk c16 (0..15) of row r in a [128][128] bf16 operand
@@ -149,20 +138,14 @@ JF_DEV uint32_t tc_swz(int r, int c16) {
   return (uint32_t)((c16 >> 3) * TC_BLK + r * 128 + (((c16 & 7) ^ (r & 7)) << 4));
 }
 
-JF_DEV void stsm_x4_t(uint32_t addr, uint32_t r0, uint32_t r1, uint32_t r2, uint32_t r3) {
-  asm volatile("stmatrix.sync.aligned.m8n8.x4.trans.shared.b16 [%0], {%1,%2,%3,%4};" ::"r"(addr), "r"(r0), "r"(r1),
-               "r"(r2), "r"(r3)
-               : "memory");
-}
-
 // K and V rows of `chunk` into one stage ({K, V} in the operand layout); `part` selects the
 // cached (1) and / or in-flight (2) keys.
 JF_DEV void issue_kv_tc(const AttnParams& a, const AttnUnit& u, int chunk, int li, int max_kp, const int* s_page,
                         uint32_t stage, int part) {
   const bf16* Kp = reinterpret_cast<const bf16*>(a.k_pages);
-  const bf16* Vp = reinterpret_cast<const bf16*>(a.v_pages);
+  const __half* Vp = reinterpret_cast<const __half*>(a.v_pages);  // V is stored in fp16
   const bf16* Ki = reinterpret_cast<const bf16*>(a.k_inf);
-  const bf16* Vi = reinterpret_cast<const bf16*>(a.v_inf);
+  const __half* Vi = reinterpret_cast<const __half*>(a.v_inf);
   const int kp0 = chunk * kAttnChunk;
   for (int i = threadIdx.x; i < kAttnChunk * 16; i += blockDim.x) {
     const int r = i >> 4, c = i & 15;
@@ -170,7 +153,7 @@ JF_DEV void issue_kv_tc(const AttnParams& a, const AttnUnit& u, int chunk, int l
     const bool cached = kp < u.pos0;
     if (!(part & (cached ? 1 : 2))) continue;
     const bf16* kr = nullptr;
-    const bf16* vr = nullptr;
+    const __half* vr = nullptr;
     if (kp <= max_kp) {
       if (cached) {
         const int page = s_page[li * (kAttnChunk / kPage) + (r >> 4)];
@@ -191,28 +174,12 @@ JF_DEV void issue_kv_tc(const AttnParams& a, const AttnUnit& u, int chunk, int l
   }
 }
 
-// V [key][dim] (bf16) -> V^T [dim][key] (fp16, the P V operand), 8x8 blocks: warp w moves items
-// w, w+8, ... of (8 keys x 32 dims).
-JF_DEV void transpose_v(uint32_t sv, uint32_t svt, int warp, int lane) {
-  const int m = lane >> 3, rr = lane & 7;
-#pragma unroll
-  for (int it = 0; it < 8; ++it) {
-    const int item = warp + 8 * it;           // 0..63
-    const int key0 = (item >> 2) * 8, dim0 = (item & 3) * 32;
-    uint32_t r0, r1, r2, r3;
-    ldsm_x4(sv + tc_swz(key0 + rr, (dim0 >> 3) + m), r0, r1, r2, r3);
-    const int dim = dim0 + 8 * m + rr;        // destination row of this lane
-    stsm_x4_t(svt + tc_swz(dim, key0 >> 3), bf16x2_to_f16x2(r0), bf16x2_to_f16x2(r1), bf16x2_to_f16x2(r2),
-              bf16x2_to_f16x2(r3));
-  }
-}
-
 // At most 200 registers a thread, like the mma.sync kernel, so that its clusters are placed while
 // the QKV finish kernel's CTAs are still resident.
 __global__ void __maxnreg__(200) k_attn_tc(const AttnParams a) {
   extern __shared__ uint8_t sm_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~uintptr_t(1023));
-  const uint32_t sQ = smem_u32(sm + TC_OFF_Q), sStage = smem_u32(sm + TC_OFF_STAGE), sVt = smem_u32(sm + TC_OFF_VT);
+  const uint32_t sQ = smem_u32(sm + TC_OFF_Q), sStage = smem_u32(sm + TC_OFF_STAGE);
   __shared__ __align__(8) uint64_t bars[2];                   // S ready, P V ready
   __shared__ uint32_t tmem_slot;
   __shared__ int s_rowpos[kAttnQRows];
@@ -285,7 +252,7 @@ __global__ void __maxnreg__(200) k_attn_tc(const AttnParams a) {
   const int pos_r = s_rowpos[r];
   const uint32_t t_row = tmem + ((uint32_t)(quad * 32) << 16);
   constexpr uint32_t idesc = idesc_bf16_f32(128, 128);
-  constexpr uint32_t idesc_pv = idesc_f16_f32(128, 128);  // P V: fp16 P and fp16 V^T
+  constexpr uint32_t idesc_pv = idesc_f16_f32(128, 128) | (1u << 16);  // P V: fp16 P, fp16 V MN-major
   float o[64];
 #pragma unroll
   for (int i = 0; i < 64; ++i) o[i] = 0.f;
@@ -295,10 +262,8 @@ __global__ void __maxnreg__(200) k_attn_tc(const AttnParams a) {
   for (int t = 0; t < n_steps && ok; ++t) {
     if (t + 1 < n_steps) cp_async_wait<1>();
     else cp_async_wait<0>();
-    __syncthreads();
     const uint32_t sK = sStage + (uint32_t)((t & 1) * TC_STAGE), sV = sK + TC_OPND;
-    transpose_v(sV, sVt, warp, lane);
-    fence_proxy_async_smem();  // cp.async and stmatrix writes -> tensor-core operand reads
+    fence_proxy_async_smem();  // this thread's cp.async writes -> tensor-core operand reads
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -310,7 +275,7 @@ __global__ void __maxnreg__(200) k_attn_tc(const AttnParams a) {
       }
       tc_commit(s_full);
     }
-    if (!mbar_wait_bounded(s_full, (uint32_t)(t & 1), JF_WAIT_LIMIT_NS)) {
+    if (!mbar_wait_bounded(s_full, (uint32_t)(t & 1), a.wait_ns)) {
       if (tid == 0) jf_set_error(a.err, JF_DERR_TIMEOUT_MMA);
       ok = false;
     }
@@ -370,11 +335,13 @@ __global__ void __maxnreg__(200) k_attn_tc(const AttnParams a) {
 #pragma unroll
       for (int kk = 0; kk < 8; ++kk) {
         const uint32_t off = (uint32_t)((kk >> 2) * TC_BLK + (kk & 3) * 32);
-        tc_mma_bf16(tmem + 128, sdesc_k_sw128(sK + off), sdesc_k_sw128(sVt + off), idesc_pv, kk > 0 ? 1u : 0u);
+        // keys 16kk .. 16kk+15 of V: 16 rows of 128 bytes; the two 64-dim atoms are a block apart
+        tc_mma_bf16(tmem + 128, sdesc_k_sw128(sK + off), sdesc_mn_sw128(sV + (uint32_t)kk * 2048u, TC_BLK),
+                    idesc_pv, kk > 0 ? 1u : 0u);
       }
       tc_commit(o_full);
     }
-    if (!mbar_wait_bounded(o_full, (uint32_t)(t & 1), JF_WAIT_LIMIT_NS)) {
+    if (!mbar_wait_bounded(o_full, (uint32_t)(t & 1), a.wait_ns)) {
       if (tid == 0) jf_set_error(a.err, JF_DERR_TIMEOUT_MMA);
       ok = false;
     }
@@ -389,7 +356,7 @@ __global__ void __maxnreg__(200) k_attn_tc(const AttnParams a) {
       for (int i = 0; i < 32; ++i) o[32 + i] = o[32 + i] * al + t32[i];
     }
     tc_fence_before();
-    ok = __syncthreads_and(ok) != 0;  // the stage, V^T and both TMEM accumulators are free again
+    ok = __syncthreads_and(ok) != 0;  // the stage and both TMEM accumulators are free again
     if (t + 2 < n_steps) {
       issue_kv_tc(a, u, sub_of(t + 2), t + 2, max_kp, s_page, sK, 3);
       cp_async_commit();

@@ -119,7 +119,6 @@ JF_DEV bool mbar_wait_bounded(uint32_t bar, uint32_t parity, uint64_t limit_ns) 
   }
 }
 
-constexpr uint64_t JF_WAIT_LIMIT_NS = 2000000000ull;  // 2 s: far beyond any legitimate wait
 
 // ------------------------------------------------------------------------------------------
 // Thread-block clusters: ranks, cluster-wide barrier
@@ -232,6 +231,19 @@ JF_DEV uint64_t sdesc_k_sw128(uint32_t saddr) {
   uint64_t d = 0;
   d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
   d |= (uint64_t)(16u >> 4) << 16;
+  d |= (uint64_t)(1024u >> 4) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+
+// Shared-memory descriptor of an MN-major operand with the 128-byte swizzle: rows of 64 MN
+// elements (128 bytes) at consecutive K indices, swizzled in 8-row groups 1024 bytes apart (stride
+// byte offset); consecutive 64-element MN atoms `lbo` bytes apart (leading byte offset).
+JF_DEV uint64_t sdesc_mn_sw128(uint32_t saddr, uint32_t lbo) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
   d |= (uint64_t)(1024u >> 4) << 32;
   d |= (uint64_t)1 << 46;
   d |= (uint64_t)2 << 61;

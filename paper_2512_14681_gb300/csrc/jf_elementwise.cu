@@ -126,6 +126,16 @@ __device__ __forceinline__ void ldcg4x4(const float* p, size_t stride, int n, fl
 }
 
 __device__ __forceinline__ void store4(float* y, float4 v) { *reinterpret_cast<float4*>(y) = v; }
+// four values rounded to bf16, then converted to fp16 (exact for magnitudes in [2^-14, 65504];
+// smaller ones keep fp16's subnormal spacing 2^-24), stored as fp16 bit patterns
+__device__ __forceinline__ void store4_bf16_as_f16(bf16* y, float4 v) {
+  const __half2 lo = __floats2half2_rn(__bfloat162float(__float2bfloat16_rn(v.x)),
+                                       __bfloat162float(__float2bfloat16_rn(v.y)));
+  const __half2 hi = __floats2half2_rn(__bfloat162float(__float2bfloat16_rn(v.z)),
+                                       __bfloat162float(__float2bfloat16_rn(v.w)));
+  *reinterpret_cast<uint2*>(y) = make_uint2(*reinterpret_cast<const uint32_t*>(&lo),
+                                            *reinterpret_cast<const uint32_t*>(&hi));
+}
 __device__ __forceinline__ void store4(bf16* y, float4 v) {
   const uint32_t lo = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.x)) |
                       ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.y)) << 16);
@@ -212,7 +222,7 @@ __global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(float* __restrict__ x,
 // tile per head): for row m and head slot hs (query heads, then key heads, then value heads), add
 // the partials in split order, rotate query and key heads by the row's position (rotate-half RoPE,
 // the same arithmetic as the fused epilogue), round to bf16 and store to q [m][Hq][128],
-// k / v [m][Hkv][128]. One warp per (row, head slot); lane l holds dims 4l .. 4l+3, whose rotation
+// k / v [m][Hkv][128] (v as fp16 values of the bf16-rounded numbers). One warp per (row, head slot); lane l holds dims 4l .. 4l+3, whose rotation
 // partner is lane l ^ 16.
 __global__ void __launch_bounds__(128) k_qkv_finish(SplitPartials sp, const int* __restrict__ pos,
                                                      const float2* __restrict__ rope, bf16* __restrict__ q,
@@ -258,10 +268,13 @@ __global__ void __launch_bounds__(128) k_qkv_finish(SplitPartials sp, const int*
       a = make_float4(a.x * c0.x + b.x * c0.y, a.y * c1.x + b.y * c1.y, a.z * c2.x + b.z * c2.y, a.w * c3.x + b.w * c3.y);
     }
     dst = (hs < Hq) ? q + ((size_t)m * Hq + hs) * 128 : k + ((size_t)m * Hkv + (hs - Hq)) * 128;
+    store4(dst + lane * 4, a);
   } else {
+    // values: rounded to bf16 (the model's rounding point), then stored as fp16, the type the
+    // attention's P V product reads them in (exact for magnitudes in fp16's normal range)
     dst = v + ((size_t)m * Hkv + (hs - Hq - Hkv)) * 128;
+    store4_bf16_as_f16(dst + lane * 4, a);
   }
-  store4(dst + lane * 4, a);
   JF_TL_EXIT(TL_QKV_FINISH);
 }
 
@@ -284,6 +297,26 @@ cudaError_t launch_pdl(K kernel, dim3 grid, dim3 block, cudaStream_t st, Args...
 #ifdef JF_TIMELINE
 JF_TL_SETTER(tl_set_elem)
 #endif
+
+// Wait-limit probe: one thread waits, under the given limit, on a shared-memory mbarrier that
+// nothing arrives at (no copy and no MMA is in flight), then stores how long it waited, records
+// JF_DERR_TIMEOUT_PROBE in the error word and exits. It exercises the same bounded wait and
+// error path as the kernels' waits on copies and MMAs, without leaving any operation behind.
+__global__ void k_wait_probe(int* err, unsigned long long* waited_ns, unsigned long long limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  const uint32_t b = smem_u32(&bar);
+  mbar_init(b, 1);
+  fence_mbar_init();
+  const uint64_t t0 = jf_globaltimer();
+  const bool arrived = mbar_wait_bounded(b, 0u, limit_ns);
+  *waited_ns = jf_globaltimer() - t0;
+  if (!arrived) jf_set_error(err, JF_DERR_TIMEOUT_PROBE);
+}
+
+cudaError_t launch_wait_probe(int* err, unsigned long long* waited_ns, unsigned long long limit_ns, cudaStream_t st) {
+  k_wait_probe<<<1, 1, 0, st>>>(err, waited_ns, limit_ns);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_init_weights(void* dst, bool is_bf16, long long rows, long long cols, uint64_t seed, uint64_t tid,
                                 double stdv, long long grp, long long grp_stride, long long grp_off, cudaStream_t st) {

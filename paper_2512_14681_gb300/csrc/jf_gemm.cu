@@ -480,7 +480,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         for (int kb = w.kb0; kb < w.kb1; ++kb, ++j) {
           if (j < pre) continue;
           const int s = j % S;
-          if (!mbar_wait_bounded(empty0 + 8 * s, (uint32_t)((j / S) - 1) & 1u, JF_WAIT_LIMIT_NS)) {
+          if (!mbar_wait_bounded(empty0 + 8 * s, (uint32_t)((j / S) - 1) & 1u, p.wait_ns)) {
             jf_set_error(p.err, JF_DERR_TIMEOUT_MMA);
             ok = false;
             break;
@@ -500,7 +500,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       for (int u = blockIdx.x; u < total_units && ok; u += gridDim.x, ++i) {
         const Unit w = unit_of(p, u);
         const int acc = i & 1;
-        if (i >= 2 && !mbar_wait_bounded(tempty0 + 8 * acc, (uint32_t)((i >> 1) - 1) & 1u, JF_WAIT_LIMIT_NS)) {
+        if (i >= 2 && !mbar_wait_bounded(tempty0 + 8 * acc, (uint32_t)((i >> 1) - 1) & 1u, p.wait_ns)) {
           jf_set_error(p.err, JF_DERR_TIMEOUT_EPI);
           break;
         }
@@ -508,7 +508,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         const uint32_t dacc = tmem + (uint32_t)(acc * Cfg::ACC_COLS);
         for (int kb = w.kb0; kb < w.kb1; ++kb, ++j) {
           const int s = j % S;
-          if (!mbar_wait_bounded(full0 + 8 * s, (uint32_t)(j / S) & 1u, JF_WAIT_LIMIT_NS)) {
+          if (!mbar_wait_bounded(full0 + 8 * s, (uint32_t)(j / S) & 1u, p.wait_ns)) {
             jf_set_error(p.err, JF_DERR_TIMEOUT_TMA);
             ok = false;
             break;
@@ -537,7 +537,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     for (int u = blockIdx.x; u < total_units; u += gridDim.x, ++i) {
       const Unit w = unit_of(p, u);
       const int acc = i & 1;
-      if (!mbar_wait_bounded(tfull0 + 8 * acc, (uint32_t)(i >> 1) & 1u, JF_WAIT_LIMIT_NS)) {
+      if (!mbar_wait_bounded(tfull0 + 8 * acc, (uint32_t)(i >> 1) & 1u, p.wait_ns)) {
         jf_set_error(p.err, JF_DERR_TIMEOUT_EPI);
         break;
       }

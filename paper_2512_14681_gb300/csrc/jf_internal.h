@@ -15,7 +15,14 @@ enum DeviceError : int {
   JF_DERR_TIMEOUT_EPI = 3,   // the accumulator barrier never completed
   JF_DERR_BOUNDS = 4,        // a page-table / token / position index was out of range
   JF_DERR_STATE = 5,         // inconsistent decode state detected on the device
+  JF_DERR_TIMEOUT_PROBE = 6, // the wait-limit probe's wait ran out (its intended outcome)
 };
+
+// Default limit of every bounded device wait: far beyond any legitimate wait. A context's limit
+// is host-settable within [kWaitLimitMinNs, kWaitLimitMaxNs].
+constexpr unsigned long long kWaitLimitDefaultNs = 2000000000ull;  // 2 s
+constexpr unsigned long long kWaitLimitMinNs = 1000000ull;         // 1 ms
+constexpr unsigned long long kWaitLimitMaxNs = 60000000000ull;     // 60 s
 
 
 constexpr int kPage = 16;         // tokens per KV page
@@ -90,6 +97,7 @@ struct GemmParams {
   float* ws;           // split-K partials [n_tiles][m_tiles][k_splits][BN][128]
   int* tile_counter;   // [m_tiles*n_tiles], zero between launches
   int* err;
+  unsigned long long wait_ns;  // limit of each bounded wait
   GemmEpi epi;
 };
 
@@ -109,6 +117,7 @@ struct AttnParams {
   int Hq, Hkv, hd;
   float scale_log2;     // log2(e) / sqrt(hd)
   int* err;
+  unsigned long long wait_ns;  // limit of each bounded wait
   float* xchg;          // bf16 path: lane states [unit][lane][kAttnXchgFloats]
 };
 

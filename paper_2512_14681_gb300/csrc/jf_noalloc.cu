@@ -80,6 +80,7 @@ extern "C" jf_status jf_op_gemm_noalloc(const void* W, const void* X, float* Y, 
   p.ws = reinterpret_cast<float*>(scratch);
   p.tile_counter = tickets;
   p.err = err_word;
+  p.wait_ns = kWaitLimitDefaultNs;
   p.epi.kind = EPI_STORE;
   p.epi.M = M;
   p.epi.N = N;

@@ -28,6 +28,7 @@ cudaError_t launch_qkv_finish(const SplitPartials& sp, const int* pos, const flo
                               int M, int Hq, int Hkv, cudaStream_t st);
 cudaError_t launch_attn_tc(const AttnParams& a, int units_bound, cudaStream_t st);
 cudaError_t launch_attn_f32(const AttnParams& a, int n_rows, cudaStream_t st);
+cudaError_t launch_wait_probe(int* err, unsigned long long* waited_ns, unsigned long long limit_ns, cudaStream_t st);
 cudaError_t gemm_prepare();
 cudaError_t attn_prepare();
 }  // namespace jf
@@ -318,6 +319,7 @@ struct jf_ctx {
   std::vector<cudaEvent_t>* capture_events = nullptr;
   std::vector<int>* capture_classes = nullptr;
   long long launches = 0;  // libjf kernels launched (graph replays count their kernel nodes)
+  unsigned long long wait_ns = kWaitLimitDefaultNs;  // limit of each bounded device wait
 };
 
 namespace {
@@ -340,7 +342,8 @@ T* at(jf_ctx* c, size_t off) {
 
 jf_status check_err_word(jf_ctx* c, int code) {
   if (code == 0) return JF_OK;
-  if (code == JF_DERR_TIMEOUT_TMA || code == JF_DERR_TIMEOUT_MMA || code == JF_DERR_TIMEOUT_EPI)
+  if (code == JF_DERR_TIMEOUT_TMA || code == JF_DERR_TIMEOUT_MMA || code == JF_DERR_TIMEOUT_EPI ||
+      code == JF_DERR_TIMEOUT_PROBE)
     return fail(c, JF_ETIMEOUT, "device wait timed out (code " + std::to_string(code) + ")");
   return fail(c, JF_EDEVICE, "device bounds check failed (code " + std::to_string(code) + ")");
 }
@@ -443,6 +446,7 @@ cudaError_t gemm(jf_ctx* c, const CUtensorMap& tmA, const void* W, const void* X
   p.ws = c->gemm_ws;
   p.tile_counter = c->gemm_counter;
   p.err = c->err;
+  p.wait_ns = c->wait_ns;
   p.grid = c->num_sms;
   p.epi = epi;
   p.epi.M = M;
@@ -514,6 +518,7 @@ cudaError_t enqueue_forward(jf_ctx* c, int M, LmMode lm) {
     a.out = c->att; a.Hq = D.Hq; a.Hkv = D.Hkv; a.hd = D.hd;
     a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)D.hd));
     a.err = c->err;
+    a.wait_ns = c->wait_ns;
     a.xchg = c->attn_xchg;
     prof_begin(c, PC_ATTN);
     if (D.bf16) {
@@ -1448,6 +1453,30 @@ jf_status jf_set_profiling(jf_ctx* c, int enable) {
   return JF_OK;
 }
 
+jf_status jf_set_wait_limit(jf_ctx* c, uint64_t limit_ns) {
+  if (!c) return JF_EINVAL;
+  if (limit_ns < kWaitLimitMinNs || limit_ns > kWaitLimitMaxNs)
+    return fail(c, JF_EINVAL, "wait limit outside [1 ms, 60 s]");
+  if (limit_ns != c->wait_ns) {
+    c->wait_ns = limit_ns;
+    drop_graphs(c);  // the iteration graphs hold the old limit in their kernel parameters
+  }
+  return JF_OK;
+}
+
+jf_status jf_wait_limit_probe(jf_ctx* c, uint64_t* waited_ns) {
+  if (!c) return JF_EINVAL;
+  // bytes 8..15 of the error slot receive the time the probe waited
+  unsigned long long* waited_dev = reinterpret_cast<unsigned long long*>(c->err + 2);
+  CK(launch_wait_probe(c->err, waited_dev, c->wait_ns, c->st));
+  c->launches += 1;
+  unsigned long long w = 0;
+  CK(cudaMemcpyAsync(&w, waited_dev, sizeof(w), cudaMemcpyDeviceToHost, c->st));
+  const jf_status s = read_err(c);  // synchronises the stream: the probe has exited
+  if (waited_ns) *waited_ns = w;
+  return s;
+}
+
 jf_status jf_tl_enable(void* records, void* counter) {
 #ifdef JF_TIMELINE
   if ((records == nullptr) != (counter == nullptr)) return JF_EINVAL;
@@ -1517,6 +1546,7 @@ jf_status jf_op_gemm(int dtype, const void* W, const void* X, float* Y, int N, i
   p.ws = reinterpret_cast<float*>(workspace);
   p.tile_counter = workspace ? reinterpret_cast<int*>(reinterpret_cast<char*>(workspace) + rup(partial, 256)) : nullptr;
   p.err = err_word;
+  p.wait_ns = kWaitLimitDefaultNs;
   p.epi.kind = EPI_STORE;
   p.epi.M = M;
   p.epi.N = N;

@@ -248,6 +248,16 @@ class Context:
         self._c(self.lib.jf_kernel_time(self.h, cls, C.byref(ms), C.byref(n)))
         return ms.value, n.value
 
+    def set_wait_limit(self, limit_ns: int):
+        """Limit of every bounded device wait of this context (jf_set_wait_limit)."""
+        self._c(self.lib.jf_set_wait_limit(self.h, int(limit_ns)))
+
+    def wait_limit_probe(self):
+        """(status, waited ns) of jf_wait_limit_probe; JF_ETIMEOUT is its expected status."""
+        w = C.c_uint64()
+        st = self.lib.jf_wait_limit_probe(self.h, C.byref(w))
+        return st, w.value
+
 
 def op_gemm(W, X, k_splits: int = 0, stream=None):
     """Y = X W^T through jf_op_gemm (torch CUDA tensors W [N,K], X [M,K], bf16 or fp32)."""

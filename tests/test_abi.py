@@ -123,6 +123,8 @@ def test_null_context_is_refused_without_touching_a_device(lib):
         "jf_generate_device": (None, 1, None, one, C.byref(gp), None, None),
         "jf_set_profiling": (None, 1),
         "jf_kernel_time": (None, 0, C.byref(d), C.byref(ll)),
+        "jf_set_wait_limit": (None, 2_000_000_000),
+        "jf_wait_limit_probe": (None, None),
     }
     for name, args in calls.items():
         assert getattr(lib, name)(*args) == J.JF_EINVAL, name

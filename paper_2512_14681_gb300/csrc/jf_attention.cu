@@ -11,14 +11,16 @@
 //
 // bf16 path: split-KV flash decoding on the tcgen05 tensor cores with a fixed reduction tree.
 // Work unit = (chain, KV head, tile of 128 (token, head) query rows). Key positions are cut into
-// absolute 128-key chunks, and chunk c belongs to lane c mod 8. A unit runs on one 8-CTA cluster:
+// absolute 128-key chunks, and chunk c belongs to lane c mod 8. A unit runs on 8 CTAs (an 8-CTA
+// cluster while all units' clusters fit on the GPU at once, independent CTAs beyond that):
 // CTA j walks the chunks of lane j in increasing order with one online-softmax state per row:
 // S = Q K^T into tensor memory, the softmax step read straight out of it, P (fp16) back to shared
 // memory, P V (fp16 operands; the cache holds V in fp16) into a second tensor-memory accumulator
 // added into registers. K/V rows are staged by cp.async (the next chunk in flight while the
 // current one computes). Each CTA then writes its
 // lane state (O, running max, sum) to a global scratch slot of the unit; after a cluster barrier
-// CTA j folds rows 16j .. 16j+15 over the 8 lanes in lane order. The tree depends only on
+// CTA j folds rows 16j .. 16j+15 over the 8 lanes in lane order (unclustered: the last lane to
+// finish folds all rows, in the same order). The tree depends only on
 // absolute key positions, never on how many rows share the forward or how many chunks a unit
 // has, so a row's result is the same in every batch.
 // fp32 path: one warp per (row, head), keys in absolute order, online softmax in fp32.
@@ -174,8 +176,51 @@ JF_DEV void issue_kv_tc(const AttnParams& a, const AttnUnit& u, int chunk, int l
   }
 }
 
+// Fold of rows rb*16 .. rb*16+15 of unit ui over its 8 lane states in lane order (thread: row
+// tid % 16, dims 8 (tid / 16) ..), normalised and stored in bf16. The same arithmetic whichever CTA
+// of the unit runs it.
+JF_DEV void fold_row_block(const AttnParams& a, const AttnUnit& u, int ui, int rb, int qr0, int qrows, int G, int tid) {
+  const int lr = tid & 15, rw = rb * ROWS_PER_CTA + lr;
+  const int d = (tid >> 4) * 8;
+  if (rw >= qrows) return;
+  const float* x0 = a.xchg + (size_t)ui * kAttnLanes * kAttnXchgFloats;
+  float ov[kAttnLanes][8], mv[kAttnLanes], lv[kAttnLanes];
+#pragma unroll
+  for (int q = 0; q < kAttnLanes; ++q) {
+    const float* xq = x0 + (size_t)q * kAttnXchgFloats;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) ov[q][e] = __ldcg(xq + (d + e) * kAttnQRows + rw);
+    mv[q] = __ldcg(xq + HD * kAttnQRows + rw);
+    lv[q] = __ldcg(xq + HD * kAttnQRows + kAttnQRows + rw);
+  }
+  float M = mv[0], L = lv[0];
+  float acc[8];
+#pragma unroll
+  for (int e = 0; e < 8; ++e) acc[e] = ov[0][e];
+#pragma unroll
+  for (int q = 1; q < kAttnLanes; ++q) {
+    float wa, wb, mm;
+    fold_weights(M, mv[q], wa, wb, mm);
+    M = mm;
+    L = wa * L + wb * lv[q];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) acc[e] = wa * acc[e] + wb * ov[q][e];
+  }
+  const float il = L > 0.f ? 1.f / L : 0.f;
+  const int qr = qr0 + rw, tq = qr / G, g = qr % G;
+  bf16* dst = reinterpret_cast<bf16*>(a.out) + ((size_t)(u.row0 + tq) * a.Hq + u.kvh * G + g) * HD + d;
+  *reinterpret_cast<uint4*>(dst) = make_uint4(pack_bf16(acc[0] * il, acc[1] * il), pack_bf16(acc[2] * il, acc[3] * il),
+                                              pack_bf16(acc[4] * il, acc[5] * il), pack_bf16(acc[6] * il, acc[7] * il));
+}
+
+// kCluster: a unit's 8 lanes run as one 8-CTA cluster and, after a cluster barrier, CTA j folds
+// rows 16j .. 16j+15 (the fastest fold; at most 15 such clusters of this kernel are resident on the
+// 152 SMs at once). Otherwise the lanes are independent CTAs (all SMs usable) and the last lane of
+// a unit to finish, found by a per-unit ticket, folds all 128 rows and resets the ticket. Both
+// forms fold in lane order with the same arithmetic, so their results are bit-identical.
 // At most 200 registers a thread, like the mma.sync kernel, so that its clusters are placed while
 // the QKV finish kernel's CTAs are still resident.
+template <bool kCluster>
 __global__ void __maxnreg__(200) k_attn_tc(const AttnParams a) {
   extern __shared__ uint8_t sm_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~uintptr_t(1023));
@@ -187,11 +232,12 @@ __global__ void __maxnreg__(200) k_attn_tc(const AttnParams a) {
   __shared__ AttnUnit s_unit;
   __shared__ float red_max[2][kAttnQRows];
   __shared__ float red_l[2][kAttnQRows];
+  __shared__ int s_last;
 
   JF_TL_ENTRY();
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int j = (int)cluster_rank();
-  const int ui = (int)cluster_id_x();
+  const int j = (int)(blockIdx.x % kAttnLanes);  // = rank in the cluster when clustered
+  const int ui = (int)(blockIdx.x / kAttnLanes);
   const int G = a.Hq / a.Hkv;
   const uint32_t s_full = smem_u32(&bars[0]), o_full = smem_u32(&bars[1]);
   pdl_launch_dependents();  // the next kernel may launch now
@@ -202,7 +248,7 @@ __global__ void __maxnreg__(200) k_attn_tc(const AttnParams a) {
   }
   resolve_unit(a, ui, j, G, warp, lane, s_unit);
   const AttnUnit u = s_unit;
-  if (!u.pad) return;  // past the last unit: the whole cluster leaves together
+  if (!u.pad) return;  // past the last unit: the whole unit (cluster) leaves together
   if (warp == 0) {
     tmem_alloc(smem_u32(&tmem_slot), TC_TMEM_COLS);
     tmem_relinquish();
@@ -365,7 +411,8 @@ __global__ void __maxnreg__(200) k_attn_tc(const AttnParams a) {
   cp_async_wait<0>();
   // lane state of the 128 rows (O, m, l over both column halves) to this lane's slot of the
   // unit in global memory, O stored dimension-major ([dim][row]: a warp writes 128 contiguous
-  // bytes per dimension); after the cluster barrier CTA j folds rows 16j .. 16j+15.
+  // bytes per dimension); then the fold (CTA j: rows 16j .. 16j+15 after the cluster barrier, or
+  // the unit's last lane: all rows).
   red_l[half][r] = l_run;
   __syncthreads();
   float* xs = a.xchg + ((size_t)ui * kAttnLanes + j) * kAttnXchgFloats;
@@ -375,39 +422,19 @@ __global__ void __maxnreg__(200) k_attn_tc(const AttnParams a) {
     xs[HD * kAttnQRows + r] = m_run;
     xs[HD * kAttnQRows + kAttnQRows + r] = red_l[0][r] + red_l[1][r];
   }
-  cluster_sync();  // release / acquire: every lane's state of the unit is visible
-  {
-    const int lr = tid & 15, rw = j * ROWS_PER_CTA + lr;
-    const int d = (tid >> 4) * 8;
-    if (ok && rw < qrows) {
-      const float* x0 = a.xchg + (size_t)ui * kAttnLanes * kAttnXchgFloats;
-      float ov[kAttnLanes][8], mv[kAttnLanes], lv[kAttnLanes];
-#pragma unroll
-      for (int q = 0; q < kAttnLanes; ++q) {
-        const float* xq = x0 + (size_t)q * kAttnXchgFloats;
-#pragma unroll
-        for (int e = 0; e < 8; ++e) ov[q][e] = __ldcg(xq + (d + e) * kAttnQRows + rw);
-        mv[q] = __ldcg(xq + HD * kAttnQRows + rw);
-        lv[q] = __ldcg(xq + HD * kAttnQRows + kAttnQRows + rw);
-      }
-      float M = mv[0], L = lv[0];
-      float acc[8];
-#pragma unroll
-      for (int e = 0; e < 8; ++e) acc[e] = ov[0][e];
-#pragma unroll
-      for (int q = 1; q < kAttnLanes; ++q) {
-        float wa, wb, mm;
-        fold_weights(M, mv[q], wa, wb, mm);
-        M = mm;
-        L = wa * L + wb * lv[q];
-#pragma unroll
-        for (int e = 0; e < 8; ++e) acc[e] = wa * acc[e] + wb * ov[q][e];
-      }
-      const float il = L > 0.f ? 1.f / L : 0.f;
-      const int qr = qr0 + rw, tq = qr / G, g = qr % G;
-      bf16* dst = reinterpret_cast<bf16*>(a.out) + ((size_t)(u.row0 + tq) * a.Hq + u.kvh * G + g) * HD + d;
-      *reinterpret_cast<uint4*>(dst) = make_uint4(pack_bf16(acc[0] * il, acc[1] * il), pack_bf16(acc[2] * il, acc[3] * il),
-                                                  pack_bf16(acc[4] * il, acc[5] * il), pack_bf16(acc[6] * il, acc[7] * il));
+  if constexpr (kCluster) {
+    cluster_sync();  // release / acquire: every lane's state of the unit is visible
+    if (ok) fold_row_block(a, u, ui, j, qr0, qrows, G, tid);
+  } else {
+    __threadfence();  // this lane's state, then its ticket
+    __syncthreads();
+    if (tid == 0) s_last = atomicAdd(a.unit_ticket + ui, 1) == kAttnLanes - 1;
+    __syncthreads();
+    if (s_last) {
+      __threadfence();  // the other lanes' states are visible to the last one
+      if (ok)
+        for (int rb = 0; rb < kAttnLanes; ++rb) fold_row_block(a, u, ui, rb, qr0, qrows, G, tid);
+      if (tid == 0) a.unit_ticket[ui] = 0;  // ready for the next launch
     }
   }
   tc_fence_after();
@@ -493,7 +520,7 @@ __global__ void __launch_bounds__(128) k_attn_f32(const AttnParams a, int n_rows
 JF_TL_SETTER(tl_set_attn)
 #endif
 
-cudaError_t launch_attn_tc(const AttnParams& a, int units_bound, cudaStream_t st) {
+cudaError_t launch_attn_tc(const AttnParams& a, int units_bound, bool clustered, cudaStream_t st) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(kAttnLanes * units_bound);
   cfg.blockDim = dim3(ATT_THREADS);
@@ -507,12 +534,15 @@ cudaError_t launch_attn_tc(const AttnParams& a, int units_bound, cudaStream_t st
   at[1].val.clusterDim.y = 1;
   at[1].val.clusterDim.z = 1;
   cfg.attrs = at;
-  cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, k_attn_tc, a);
+  cfg.numAttrs = clustered ? 2 : 1;
+  return clustered ? cudaLaunchKernelEx(&cfg, k_attn_tc<true>, a) : cudaLaunchKernelEx(&cfg, k_attn_tc<false>, a);
 }
 
-cudaError_t attn_prepare() {
-  cudaError_t e = cudaFuncSetAttribute(k_attn_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, TC_SMEM);
+// Shared-memory limits of both forms; *max_clusters = how many 8-CTA clusters of the clustered
+// form can be resident at once (0 = none, an error).
+cudaError_t attn_prepare(int* max_clusters) {
+  cudaError_t e = cudaFuncSetAttribute(k_attn_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, TC_SMEM);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_attn_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, TC_SMEM);
   if (e != cudaSuccess) return e;
   // an 8-CTA cluster of this kernel must fit on the device
   cudaLaunchConfig_t cfg = {};
@@ -527,8 +557,9 @@ cudaError_t attn_prepare() {
   cfg.attrs = at;
   cfg.numAttrs = 1;
   int n_clusters = 0;
-  e = cudaOccupancyMaxActiveClusters(&n_clusters, k_attn_tc, &cfg);
+  e = cudaOccupancyMaxActiveClusters(&n_clusters, k_attn_tc<true>, &cfg);
   if (e != cudaSuccess) return e;
+  *max_clusters = n_clusters;
   return n_clusters > 0 ? cudaSuccess : cudaErrorInvalidConfiguration;
 }
 

@@ -119,6 +119,7 @@ struct AttnParams {
   int* err;
   unsigned long long wait_ns;  // limit of each bounded wait
   float* xchg;          // bf16 path: lane states [unit][lane][kAttnXchgFloats]
+  int* unit_ticket;     // bf16 path, unclustered form: lanes finished per unit, zero between launches
 };
 
 // Host-side launch helpers of the projection GEMM (jf_gemm.cu) and the TMA descriptor encoder

@@ -26,11 +26,11 @@ cudaError_t launch_rmsnorm(float* x, const float* gain, void* y, bool is_bf16, i
                            const SplitPartials* acc, int row0, cudaStream_t st);
 cudaError_t launch_qkv_finish(const SplitPartials& sp, const int* pos, const float2* rope, void* q, void* k, void* v,
                               int M, int Hq, int Hkv, cudaStream_t st);
-cudaError_t launch_attn_tc(const AttnParams& a, int units_bound, cudaStream_t st);
+cudaError_t launch_attn_tc(const AttnParams& a, int units_bound, bool clustered, cudaStream_t st);
 cudaError_t launch_attn_f32(const AttnParams& a, int n_rows, cudaStream_t st);
 cudaError_t launch_wait_probe(int* err, unsigned long long* waited_ns, unsigned long long limit_ns, cudaStream_t st);
 cudaError_t gemm_prepare();
-cudaError_t attn_prepare();
+cudaError_t attn_prepare(int* max_clusters);
 }  // namespace jf
 
 using namespace jf;
@@ -109,7 +109,7 @@ struct Offsets {
   std::vector<size_t> w_qkv, w_o, w_gu, w_d, g_attn, g_mlp;
   size_t k_pages, v_pages, page_table, seq_len, commit;
   size_t k_inf, v_inf, x, h, q, att, act;
-  size_t tok, pos, gpred, top2, chains, n_chains, attn_xchg;
+  size_t tok, pos, gpred, top2, chains, n_chains, attn_xchg, attn_ticket;
   size_t gemm_ws, gemm_counter, am_v1, am_i1, am_v2, am_counter;
   size_t logits, err, traj_count;
   size_t gen_state, gen_out, gen_truth, gen_log, gen_q0, gen_plast, gen_prompt, gen_seqp, res, step_blocks, step_res,
@@ -213,6 +213,7 @@ Offsets plan_offsets(const Dims& D) {
   o.n_chains = p.take(16);
   // attention lane states: [unit][lane][128 x 128 O, 128 m, 128 l] fp32 (bf16 path)
   o.attn_xchg = p.take(D.bf16 ? (size_t)D.max_units * kAttnLanes * kAttnXchgFloats * 4 : 16, 1024);
+  o.attn_ticket = p.take((size_t)D.max_units * 4);
   o.gemm_ws_bytes = gemm_ws_floats(D) * 4;
   o.gemm_ws = p.take(std::max<size_t>(o.gemm_ws_bytes, 16), 1024);
   const int max_mt = cdiv(D.R, 16) + 1;
@@ -290,6 +291,8 @@ struct jf_ctx {
   Chain* chains;
   int* n_chains;
   float* attn_xchg;
+  int* attn_ticket;
+  int attn_max_clusters = 0;  // 8-CTA clusters of the attention resident at once
   int chains_bound = 1;  // most chains the next forward can have (sizes the attention launch)
   float* gemm_ws;
   int* gemm_counter;
@@ -520,11 +523,20 @@ cudaError_t enqueue_forward(jf_ctx* c, int M, LmMode lm) {
     a.err = c->err;
     a.wait_ns = c->wait_ns;
     a.xchg = c->attn_xchg;
+    a.unit_ticket = c->attn_ticket;
     prof_begin(c, PC_ATTN);
     if (D.bf16) {
       // units of this forward are bounded by its rows: every chain adds at most one partial tile
       const int units_bound = std::min(D.max_units, D.Hkv * (cdiv((long long)M * D.G, kAttnQRows) + c->chains_bound));
-      e = launch_attn_tc(a, units_bound, c->st);
+      // The clustered form folds in parallel but holds at most attn_max_clusters units at once
+      // (15 on a GB300: 120 of 152 SMs); the unclustered form uses every SM and folds on one CTA
+      // per unit. Take the unclustered form only when it needs fewer waves of units, for the unit
+      // count of the rows spread evenly over the chains (exact for equal chains).
+      const int cb = std::max(1, c->chains_bound);
+      const int units_est = std::min(units_bound, D.Hkv * cb * (int)cdiv((long long)cdiv(M, cb) * D.G, kAttnQRows));
+      const int waves_cl = cdiv(units_est, std::max(1, c->attn_max_clusters));
+      const int waves_un = cdiv((long long)units_est * kAttnLanes, c->num_sms);
+      e = launch_attn_tc(a, units_bound, waves_cl <= waves_un, c->st);
       prof_end(c);
     } else {
       e = launch_attn_f32(a, M, c->st);
@@ -1016,6 +1028,7 @@ jf_status jf_create(const jf_model_config* model, const jf_runtime_config* rt, j
   c->top2 = at<float>(c, O.top2);
   c->chains = at<Chain>(c, O.chains);
   c->attn_xchg = at<float>(c, O.attn_xchg);
+  c->attn_ticket = at<int>(c, O.attn_ticket);
   c->n_chains = at<int>(c, O.n_chains);
   c->gemm_ws = at<float>(c, O.gemm_ws);
   c->gemm_counter = at<int>(c, O.gemm_counter);
@@ -1053,6 +1066,7 @@ jf_status jf_create(const jf_model_config* model, const jf_runtime_config* rt, j
   zero(O.gemm_counter, (O.am_v1 - O.gemm_counter));
   zero(O.am_counter, (size_t)(cdiv(D.R, 16) + 1) * 4);
   zero(O.err, 16);
+  zero(O.attn_ticket, (size_t)D.max_units * 4);
   zero(O.n_chains, 16);
   zero(O.x, (size_t)D.R * D.d * 4);
   zero(O.h, (size_t)D.R * D.d * D.es);
@@ -1061,7 +1075,7 @@ jf_status jf_create(const jf_model_config* model, const jf_runtime_config* rt, j
   if (e == cudaSuccess) e = cudaMemsetAsync(c->page_table, 0xff, (size_t)D.S * D.pps * 4, c->st);
   if (e == cudaSuccess) e = launch_rope_table(c->rope, D.max_ctx + 1, D.hd / 2, c->mc.rope_theta, c->st);
   if (e == cudaSuccess) e = gemm_prepare();
-  if (e == cudaSuccess) e = attn_prepare();
+  if (e == cudaSuccess) e = attn_prepare(&c->attn_max_clusters);
   if (e == cudaSuccess) e = cudaStreamSynchronize(c->st);
   if (e != cudaSuccess) return abandon(JF_ECUDA);
   *out = c;

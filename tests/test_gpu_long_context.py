@@ -8,7 +8,8 @@ partial states. Checked here:
 * a batch of three sequences with different long prompts decodes exactly as each one alone
   (a row's arithmetic does not depend on the rows in flight with it);
 * greedy Jacobi decoding equals greedy AR decoding on the device at 2540 committed tokens
-  (small model) and at 16384 committed tokens (1.5B shape).
+  (small model) and at 16384 committed tokens (1.5B shape), and with a 256-row window whose
+  attention runs the unclustered form of the kernel.
 """
 import numpy as np
 import pytest
@@ -94,5 +95,27 @@ def test_jacobi_equals_ar_16k_context_1p5b():
         ar = ctx.generate([prompt], Gen(mode="ar", max_new=24)).tokens[0]
         jac = ctx.generate([prompt], Gen(block_size=16, max_new=24)).tokens[0]
         assert np.array_equal(jac, ar)
+    finally:
+        ctx.close()
+
+
+def test_unclustered_attention_decodes_like_clustered():
+    """A 256-row Jacobi window on the small model has 16 attention units (2 KV heads x 8 query
+    tiles), more than the 15 8-CTA clusters of the attention kernel that a GB300 holds at once: as
+    clusters they take two waves, as independent CTAs (128) one, so its forwards run the unclustered
+    form (the last lane of a unit folds all its rows). AR forwards (one row, two units) run the
+    clustered form. Both fold in lane order with the same arithmetic: the tokens are identical."""
+    need_gpu()
+    from paper_2512_14681_gb300.jacobi import Context, Gen
+
+    shape = I.SMALL_BF16
+    ctx = Context(shape, max_seqs=1, max_ctx=3072, max_rows=256, logits_rows=16)
+    try:
+        ctx.init_random_weights(I.WEIGHT_SEED, I.WEIGHT_STD)
+        prompt = I.prompt_tokens(shape.vocab, P_LONG, seed=54)
+        ar = ctx.generate([prompt], Gen(mode="ar", max_new=48)).tokens[0]
+        out = ctx.generate([prompt], Gen(block_size=256, mode="window", max_new=48))
+        assert out.rows.max() == 256
+        assert np.array_equal(out.tokens[0], ar)
     finally:
         ctx.close()

@@ -48,7 +48,9 @@ typedef enum {
 
 typedef enum { JF_F32 = 0, JF_BF16 = 1 } jf_dtype;
 
-/* Decoder shape (Sec. 4.1: the Qwen2.5 family). RMSNorm -> fused QKV -> rotary embedding
+/* Decoder shape (Sec. 4.1: the Qwen2.5 family). RMSNorm -> fused QKV (+ per-feature biases when
+ * qkv_bias = 1, as in Qwen2.5; added to the projection outputs before the rotary embedding, held in
+ * the model dtype) -> rotary embedding
  * (rotate-half pairing, frequency rope_theta^(-2i/head_dim)) -> grouped-query attention ->
  * O projection + residual -> RMSNorm -> SwiGLU MLP + residual; final RMSNorm -> LM head.
  * dtype JF_BF16: weights, KV cache and matrix-product inputs are bf16; accumulation, residual
@@ -59,6 +61,8 @@ typedef struct {
   int n_layers, d_model, n_heads, n_kv_heads, head_dim, d_ff, vocab;
   double rms_eps, rope_theta;
   int dtype;
+  int qkv_bias;        /* 0 / 1: Q, K and V projections carry per-feature biases */
+  int tie_embeddings;  /* 0 / 1: the LM head is the embedding matrix (tensor 1 does not exist) */
 } jf_model_config;
 
 /* Capacity. max_rows: in-flight rows per forward (K*n + candidates, or a prefill chunk);
@@ -82,14 +86,16 @@ jf_status jf_create(const jf_model_config* model, const jf_runtime_config* rt, j
 void jf_destroy(jf_ctx* ctx);
 const char* jf_last_error(const jf_ctx* ctx);
 
-/* Weights. Logical tensors, row-major [out, in]: id 0 embedding [V,d], 1 LM head [V,d],
- * 2 final-norm gain [d]; layer l at 8+16l: +0 attention-norm gain [d], +1 Wq [Hq*hd,d],
- * +2 Wk [Hkv*hd,d], +3 Wv [Hkv*hd,d], +4 Wo [d,Hq*hd], +5 MLP-norm gain [d], +6 W_gate [F,d],
- * +7 W_up [F,d], +8 W_down [d,F].
- * jf_init_random_weights: every matrix entry = std * N(0,1) from SplitMix64 + Box-Muller keyed
- * by (seed, tensor id, element index), rounded to the model dtype; gains = 1.
- * jf_load_weights / jf_save_weights: raw file "JFW1" (header with the shape, then the tensors in
- * id order, matrices in the model dtype, gains fp32).
+/* Weights. Logical tensors, row-major [out, in]: id 0 embedding [V,d], 1 LM head [V,d] (absent
+ * with tie_embeddings), 2 final-norm gain [d]; layer l at 8+16l: +0 attention-norm gain [d],
+ * +1 Wq [Hq*hd,d], +2 Wk [Hkv*hd,d], +3 Wv [Hkv*hd,d], +4 Wo [d,Hq*hd], +5 MLP-norm gain [d],
+ * +6 W_gate [F,d], +7 W_up [F,d], +8 W_down [d,F], and with qkv_bias +9 b_q [Hq*hd],
+ * +10 b_k [Hkv*hd], +11 b_v [Hkv*hd].
+ * jf_init_random_weights: every matrix and bias entry = std * N(0,1) from SplitMix64 +
+ * Box-Muller keyed by (seed, tensor id, element index), rounded to the model dtype; gains = 1.
+ * jf_load_weights / jf_save_weights: raw file "JFW1" (header with the shape, version 2 also with
+ * qkv_bias and tie_embeddings; version-1 files load into models with neither), then the existing
+ * tensors in id order, matrices and biases in the model dtype, gains fp32).
  * jf_get_weights: copies `count` logical elements of tensor `tensor_id` from `start` into a host
  * fp32 buffer. */
 jf_status jf_init_random_weights(jf_ctx* ctx, uint64_t seed, double std);

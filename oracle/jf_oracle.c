@@ -7,9 +7,11 @@
  *
  * What it computes (Jacobi Forcing, arXiv 2512.14681):
  *   - the causal decoder-only transformer p_theta of Sec. 2.1 (Eq. 1), in the Qwen2.5 shape
- *     named in Sec. 4.1: RMSNorm -> Q/K/V -> rotary embedding -> grouped-query causal
+ *     named in Sec. 4.1: RMSNorm -> Q/K/V (+ optional per-feature biases, which the Qwen2.5
+ *     architecture has) -> rotary embedding -> grouped-query causal
  *     attention over the exact KV cache of the committed prefix -> O projection + residual
- *     -> RMSNorm -> SwiGLU MLP + residual; final RMSNorm -> LM head;
+ *     -> RMSNorm -> SwiGLU MLP + residual; final RMSNorm -> LM head (optionally the embedding
+ *     matrix itself: tied embeddings, as in the smaller Qwen2.5 models);
  *   - one forward over M in-flight rows with the block-causal ("tree") mask, which is how
  *     Eq. 3 solves all n conditionals of a Jacobi block in one pass; multi-block decoding
  *     and rejection recycling (Sec. 3.2, Algorithm 1) only add segments to this mask;
@@ -106,14 +108,18 @@ typedef struct {
     int n_layers, d_model, n_heads, n_kv_heads, head_dim, d_ff, vocab;
     double rms_eps, rope_theta;
     int bf16; /* 1: bf16 model (see header), 0: fp32 model */
+    int qkv_bias;       /* 1: Q, K and V projections carry per-feature biases */
+    int tie_embeddings; /* 1: the LM head is the embedding matrix (no tensor 1) */
 } orc_config;
 
-/* Logical tensor ids: 0 embedding [V,d], 1 LM head [V,d], 2 final-norm gain [1,d];
- * layer l at 8 + 16 l: +0 attention-norm gain [1,d], +1 Wq [Hq hd, d], +2 Wk [Hkv hd, d],
- * +3 Wv [Hkv hd, d], +4 Wo [d, Hq hd], +5 MLP-norm gain [1,d], +6 W_gate [F,d],
- * +7 W_up [F,d], +8 W_down [d,F]. Matrices are [out, in], row-major. */
+/* Logical tensor ids: 0 embedding [V,d], 1 LM head [V,d] (absent with tied embeddings),
+ * 2 final-norm gain [1,d]; layer l at 8 + 16 l: +0 attention-norm gain [1,d], +1 Wq [Hq hd, d],
+ * +2 Wk [Hkv hd, d], +3 Wv [Hkv hd, d], +4 Wo [d, Hq hd], +5 MLP-norm gain [1,d],
+ * +6 W_gate [F,d], +7 W_up [F,d], +8 W_down [d,F], and with QKV biases +9 b_q [1, Hq hd],
+ * +10 b_k [1, Hkv hd], +11 b_v [1, Hkv hd]. Matrices are [out, in], row-major; biases are
+ * held at the model's storage precision like the matrices. */
 enum { T_EMBED = 0, T_LMHEAD = 1, T_FNORM = 2 };
-enum { L_ANORM = 0, L_WQ, L_WK, L_WV, L_WO, L_MNORM, L_WG, L_WU, L_WD, L_COUNT };
+enum { L_ANORM = 0, L_WQ, L_WK, L_WV, L_WO, L_MNORM, L_WG, L_WU, L_WD, L_BQ, L_BK, L_BV, L_COUNT };
 #define ORC_LAYER_BASE 8
 #define ORC_LAYER_STRIDE 16
 
@@ -131,7 +137,7 @@ typedef struct {
 
 int orc_tensor_shape(const orc_config* c, int tid, long* rows, long* cols) {
     long d = c->d_model, qd = (long)c->n_heads * c->head_dim, kvd = (long)c->n_kv_heads * c->head_dim;
-    if (tid == T_EMBED || tid == T_LMHEAD) { *rows = c->vocab; *cols = d; return ORC_OK; }
+    if (tid == T_EMBED || (tid == T_LMHEAD && !c->tie_embeddings)) { *rows = c->vocab; *cols = d; return ORC_OK; }
     if (tid == T_FNORM) { *rows = 1; *cols = d; return ORC_OK; }
     if (tid < ORC_LAYER_BASE) return ORC_EINVAL;
     int l = (tid - ORC_LAYER_BASE) / ORC_LAYER_STRIDE, w = (tid - ORC_LAYER_BASE) % ORC_LAYER_STRIDE;
@@ -143,6 +149,8 @@ int orc_tensor_shape(const orc_config* c, int tid, long* rows, long* cols) {
         case L_WO: *rows = d; *cols = qd; break;
         case L_WG: case L_WU: *rows = c->d_ff; *cols = d; break;
         case L_WD: *rows = d; *cols = c->d_ff; break;
+        case L_BQ: if (!c->qkv_bias) return ORC_EINVAL; *rows = 1; *cols = qd; break;
+        case L_BK: case L_BV: if (!c->qkv_bias) return ORC_EINVAL; *rows = 1; *cols = kvd; break;
         default: return ORC_EINVAL;
     }
     return ORC_OK;
@@ -487,6 +495,17 @@ int orc_forward(const orc_model* m, orc_cache* c, int M, const int32_t* tokens, 
         orc_linear_t(M, h, orc_layer_t(m, l, L_WQ), q);
         orc_linear_t(M, h, orc_layer_t(m, l, L_WK), kk);
         orc_linear_t(M, h, orc_layer_t(m, l, L_WV), vv);
+        if (cf->qkv_bias) {
+            /* per-feature biases on the projection outputs, before the rotary embedding */
+            const orc_tensor *bq = orc_layer_t(m, l, L_BQ), *bk = orc_layer_t(m, l, L_BK), *bv = orc_layer_t(m, l, L_BV);
+            for (int i = 0; i < M; i++) {
+                for (int j = 0; j < qd; j++) q[(long)i * qd + j] += orc_w(bq, j);
+                for (int j = 0; j < kvd; j++) {
+                    kk[(long)i * kvd + j] += orc_w(bk, j);
+                    vv[(long)i * kvd + j] += orc_w(bv, j);
+                }
+            }
+        }
         for (int i = 0; i < M; i++) {
             for (int hh = 0; hh < Hq; hh++) orc_rope(hd, cf->rope_theta, pos[i], q + (long)i * qd + (long)hh * hd);
             for (int hh = 0; hh < Hkv; hh++) orc_rope(hd, cf->rope_theta, pos[i], kk + (long)i * kvd + (long)hh * hd);
@@ -553,7 +572,7 @@ int orc_forward(const orc_model* m, orc_cache* c, int M, const int32_t* tokens, 
         free(x); free(h); free(q); free(kk); free(vv); free(att); free(tmp); free(ut); free(gain);
         return ORC_ENOMEM;
     }
-    orc_linear_t(M, h, &m->t[T_LMHEAD], logits);
+    orc_linear_t(M, h, &m->t[cf->tie_embeddings ? T_EMBED : T_LMHEAD], logits);
     for (int i = 0; i < M; i++) {
         int a = orc_argmax_f32(V, logits + (long)i * V, top2_out ? top2_out + 2 * i : NULL);
         if (argmax_out) argmax_out[i] = a;

@@ -81,7 +81,7 @@ def _p(a, ct):
 class _Cfg(C.Structure):
     _fields_ = [("n_layers", C.c_int), ("d_model", C.c_int), ("n_heads", C.c_int), ("n_kv_heads", C.c_int),
                 ("head_dim", C.c_int), ("d_ff", C.c_int), ("vocab", C.c_int), ("rms_eps", C.c_double),
-                ("rope_theta", C.c_double), ("bf16", C.c_int)]
+                ("rope_theta", C.c_double), ("bf16", C.c_int), ("qkv_bias", C.c_int), ("tie_embeddings", C.c_int)]
 
 
 @dataclass(frozen=True)
@@ -96,16 +96,20 @@ class ModelConfig:
     rms_eps: float = 1e-6
     rope_theta: float = 1e4
     bf16: bool = False
+    qkv_bias: bool = False        # per-feature biases on the Q, K, V projections (Qwen2.5 architecture)
+    tie_embeddings: bool = False  # LM head = embedding matrix
 
     def c_struct(self) -> _Cfg:
         return _Cfg(self.n_layers, self.d_model, self.n_heads, self.n_kv_heads, self.head_dim, self.d_ff,
-                    self.vocab, self.rms_eps, self.rope_theta, int(self.bf16))
+                    self.vocab, self.rms_eps, self.rope_theta, int(self.bf16), int(self.qkv_bias),
+                    int(self.tie_embeddings))
 
 
-# Logical tensor ids (jf_oracle.c): 0 embedding, 1 LM head, 2 final-norm gain; layer l at 8+16l:
-# +0 attn-norm gain, +1 Wq, +2 Wk, +3 Wv, +4 Wo, +5 mlp-norm gain, +6 W_gate, +7 W_up, +8 W_down.
+# Logical tensor ids (jf_oracle.c): 0 embedding, 1 LM head (absent when tied), 2 final-norm gain;
+# layer l at 8+16l: +0 attn-norm gain, +1 Wq, +2 Wk, +3 Wv, +4 Wo, +5 mlp-norm gain, +6 W_gate,
+# +7 W_up, +8 W_down, and with QKV biases +9 b_q, +10 b_k, +11 b_v.
 T_EMBED, T_LMHEAD, T_FNORM = 0, 1, 2
-L_ANORM, L_WQ, L_WK, L_WV, L_WO, L_MNORM, L_WG, L_WU, L_WD = range(9)
+L_ANORM, L_WQ, L_WK, L_WV, L_WO, L_MNORM, L_WG, L_WU, L_WD, L_BQ, L_BK, L_BV = range(12)
 
 
 def layer_tid(layer: int, w: int) -> int:

@@ -41,7 +41,7 @@ class JfError(RuntimeError):
 class ModelConfig(C.Structure):
     _fields_ = [("n_layers", C.c_int), ("d_model", C.c_int), ("n_heads", C.c_int), ("n_kv_heads", C.c_int),
                 ("head_dim", C.c_int), ("d_ff", C.c_int), ("vocab", C.c_int), ("rms_eps", C.c_double),
-                ("rope_theta", C.c_double), ("dtype", C.c_int)]
+                ("rope_theta", C.c_double), ("dtype", C.c_int), ("qkv_bias", C.c_int), ("tie_embeddings", C.c_int)]
 
 
 class RuntimeConfig(C.Structure):

@@ -220,11 +220,12 @@ __global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(float* __restrict__ x,
 
 // Finish of the QKV projection from its split-K partials (EPI_PARTIAL, head_dim 128 = one weight
 // tile per head): for row m and head slot hs (query heads, then key heads, then value heads), add
-// the partials in split order, rotate query and key heads by the row's position (rotate-half RoPE,
+// the partials in split order, then the feature's bias when the model has QKV biases, rotate query and key heads by the row's position (rotate-half RoPE,
 // the same arithmetic as the fused epilogue), round to bf16 and store to q [m][Hq][128],
 // k / v [m][Hkv][128] (v as fp16 values of the bf16-rounded numbers). One warp per (row, head slot); lane l holds dims 4l .. 4l+3, whose rotation
 // partner is lane l ^ 16.
-__global__ void __launch_bounds__(128) k_qkv_finish(SplitPartials sp, const int* __restrict__ pos,
+__global__ void __launch_bounds__(128) k_qkv_finish(SplitPartials sp, const bf16* __restrict__ bias,
+                                                     const int* __restrict__ pos,
                                                      const float2* __restrict__ rope, bf16* __restrict__ q,
                                                      bf16* __restrict__ k, bf16* __restrict__ v, int M, int Hq,
                                                      int Hkv) {
@@ -253,6 +254,13 @@ __global__ void __launch_bounds__(128) k_qkv_finish(SplitPartials sp, const int*
       a.z += t[s].z;
       a.w += t[s].w;
     }
+  }
+  if (bias != nullptr) {  // per-feature bias (bf16 values), after the projection, before RoPE
+    const uint2 w = *reinterpret_cast<const uint2*>(bias + (size_t)hs * 128 + lane * 4);
+    a.x += __uint_as_float(w.x << 16);
+    a.y += __uint_as_float(w.x & 0xffff0000u);
+    a.z += __uint_as_float(w.y << 16);
+    a.w += __uint_as_float(w.y & 0xffff0000u);
   }
   bf16* dst;
   if (hs < Hq + Hkv) {
@@ -385,10 +393,11 @@ cudaError_t launch_rmsnorm(float* x, const float* gain, void* y, bool is_bf16, i
                     d, eps, sp, row0);
 }
 
-cudaError_t launch_qkv_finish(const SplitPartials& sp, const int* pos, const float2* rope, void* q, void* k, void* v,
-                              int M, int Hq, int Hkv, cudaStream_t st) {
+cudaError_t launch_qkv_finish(const SplitPartials& sp, const void* bias, const int* pos, const float2* rope, void* q,
+                              void* k, void* v, int M, int Hq, int Hkv, cudaStream_t st) {
   const int jobs = M * (Hq + 2 * Hkv);
-  return launch_pdl(k_qkv_finish, dim3((jobs + 3) / 4), dim3(128), st, sp, pos, rope, reinterpret_cast<bf16*>(q),
+  return launch_pdl(k_qkv_finish, dim3((jobs + 3) / 4), dim3(128), st, sp, reinterpret_cast<const bf16*>(bias), pos,
+                    rope, reinterpret_cast<bf16*>(q),
                     reinterpret_cast<bf16*>(k), reinterpret_cast<bf16*>(v), M, Hq, Hkv);
 }
 

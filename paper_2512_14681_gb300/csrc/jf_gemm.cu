@@ -95,8 +95,10 @@ JF_DEV void epilogue_chunk(const GemmEpi& e, const float (&v)[16], int row, int 
     }
     return;
   } else if constexpr (kind == EPI_QKV) {
+    // the feature's bias (if any) before the rotation, so that the partner reads biased values
+    const float b = (e.bias != nullptr && n < e.N) ? act_to_f32(reinterpret_cast<const T*>(e.bias)[n]) : 0.f;
 #pragma unroll
-    for (int j = 0; j < 16; ++j) xs[j * 128 + row] = v[j];
+    for (int j = 0; j < 16; ++j) xs[j * 128 + row] = v[j] + b;
     epi_sync();
     {
       const int hd = e.head_dim, half = hd >> 1;

@@ -77,6 +77,7 @@ struct GemmEpi {
   int n_q, n_kv, head_dim;
   const int* pos;
   const float2* rope;   // [max_pos][hd/2] (cos, sin)
+  const void* bias;     // per-feature Q/K/V biases [n_q + 2 n_kv] in the model dtype, added before RoPE, or null
   // EPI_SWIGLU: tile t holds features 64t..64t+63 as row pairs (gate 64t+i at 2i, up at 2i+1); act[m][64t + i]
   void* act;
   int ld_act;

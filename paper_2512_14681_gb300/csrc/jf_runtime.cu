@@ -3,6 +3,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <cstddef>
 #include <cstdio>
 #include <cstring>
 #include <map>
@@ -24,8 +25,8 @@ cudaError_t launch_embed(const void* E, bool is_bf16, const int* tok, float* x, 
                          cudaStream_t st);
 cudaError_t launch_rmsnorm(float* x, const float* gain, void* y, bool is_bf16, int rows, int d, float eps,
                            const SplitPartials* acc, int row0, cudaStream_t st);
-cudaError_t launch_qkv_finish(const SplitPartials& sp, const int* pos, const float2* rope, void* q, void* k, void* v,
-                              int M, int Hq, int Hkv, cudaStream_t st);
+cudaError_t launch_qkv_finish(const SplitPartials& sp, const void* bias, const int* pos, const float2* rope, void* q,
+                              void* k, void* v, int M, int Hq, int Hkv, cudaStream_t st);
 cudaError_t launch_attn_tc(const AttnParams& a, int units_bound, bool clustered, cudaStream_t st);
 cudaError_t launch_attn_f32(const AttnParams& a, int n_rows, cudaStream_t st);
 cudaError_t launch_wait_probe(int* err, unsigned long long* waited_ns, unsigned long long limit_ns, cudaStream_t st);
@@ -89,6 +90,7 @@ struct Dims {
   int L, d, Hq, Hkv, hd, F, V, nq, nkv, nqkv, G;
   int es;
   bool bf16;
+  bool qkv_bias, tie;  // per-feature Q/K/V biases; LM head = embedding matrix
   int R, S, max_ctx, pps, n_pages, logits_rows;
   int max_chains, max_units;
   int n_vtiles;
@@ -106,7 +108,7 @@ struct Plan {
 
 struct Offsets {
   size_t w_embed, w_lm, g_final, rope;
-  std::vector<size_t> w_qkv, w_o, w_gu, w_d, g_attn, g_mlp;
+  std::vector<size_t> w_qkv, w_o, w_gu, w_d, g_attn, g_mlp, b_qkv;
   size_t k_pages, v_pages, page_table, seq_len, commit;
   size_t k_inf, v_inf, x, h, q, att, act;
   size_t tok, pos, gpred, top2, chains, n_chains, attn_xchg, attn_ticket;
@@ -126,6 +128,10 @@ jf_status make_dims(const jf_model_config* m, const jf_runtime_config* rt, Dims*
     return JF_EINVAL;
   }
   if (m->dtype != JF_F32 && m->dtype != JF_BF16) { *why = "dtype must be JF_F32 or JF_BF16"; return JF_EINVAL; }
+  if ((m->qkv_bias != 0 && m->qkv_bias != 1) || (m->tie_embeddings != 0 && m->tie_embeddings != 1)) {
+    *why = "qkv_bias and tie_embeddings must be 0 or 1";
+    return JF_EINVAL;
+  }
   if (m->n_heads % m->n_kv_heads) { *why = "n_heads must be a multiple of n_kv_heads"; return JF_EUNSUPPORTED; }
   if (m->dtype == JF_BF16 && m->head_dim != 128) { *why = "bf16 kernels need head_dim 128"; return JF_EUNSUPPORTED; }
   if (m->dtype == JF_F32 && m->head_dim != 64 && m->head_dim != 128) { *why = "head_dim must be 64 or 128"; return JF_EUNSUPPORTED; }
@@ -148,6 +154,7 @@ jf_status make_dims(const jf_model_config* m, const jf_runtime_config* rt, Dims*
   D->F = m->d_ff; D->V = m->vocab;
   D->nq = D->Hq * D->hd; D->nkv = D->Hkv * D->hd; D->nqkv = D->nq + 2 * D->nkv; D->G = D->Hq / D->Hkv;
   D->bf16 = m->dtype == JF_BF16; D->es = D->bf16 ? 2 : 4;
+  D->qkv_bias = m->qkv_bias != 0; D->tie = m->tie_embeddings != 0;
   D->R = rt->max_rows; D->S = rt->max_seqs; D->max_ctx = rt->max_ctx;
   D->pps = cdiv(rt->max_ctx, kPage); D->n_pages = D->S * D->pps; D->logits_rows = rt->logits_rows;
   D->max_chains = std::min(kMaxChains, D->S * 5 + 1);
@@ -180,7 +187,7 @@ Offsets plan_offsets(const Dims& D) {
   Plan p;
   const size_t es = D.es;
   o.w_embed = p.take((size_t)D.V * D.d * es, 1024);
-  o.w_lm = p.take((size_t)D.V * D.d * es, 1024);
+  o.w_lm = D.tie ? o.w_embed : p.take((size_t)D.V * D.d * es, 1024);
   o.g_final = p.take((size_t)D.d * 4);
   for (int l = 0; l < D.L; ++l) {
     o.w_qkv.push_back(p.take((size_t)D.nqkv * D.d * es, 1024));
@@ -189,6 +196,7 @@ Offsets plan_offsets(const Dims& D) {
     o.w_d.push_back(p.take((size_t)D.d * D.F * es, 1024));
     o.g_attn.push_back(p.take((size_t)D.d * 4));
     o.g_mlp.push_back(p.take((size_t)D.d * 4));
+    o.b_qkv.push_back(D.qkv_bias ? p.take((size_t)D.nqkv * es) : 0);  // model dtype, q | k | v
   }
   o.rope = p.take((size_t)(D.max_ctx + 1) * (D.hd / 2) * sizeof(float2));
   const size_t kv_layer = (size_t)D.n_pages * D.Hkv * kPage * D.hd * es;
@@ -243,6 +251,7 @@ Offsets plan_offsets(const Dims& D) {
 
 struct LayerW {
   void *qkv, *o, *gu, *dn;
+  void* b_qkv;  // [nq + 2 nkv] in the model dtype, or null
   float *g_attn, *g_mlp;
   CUtensorMap tm_qkv, tm_o, tm_gu, tm_dn;
 };
@@ -505,10 +514,11 @@ cudaError_t enqueue_forward(jf_ctx* c, int M, LmMode lm) {
     ep.q_out = c->q; ep.k_out = kinf; ep.v_out = vinf;
     ep.n_q = D.nq; ep.n_kv = D.nkv; ep.head_dim = D.hd;
     ep.pos = c->pos; ep.rope = c->rope;
+    ep.bias = w.b_qkv;
     if ((e = gemm(c, w.tm_qkv, w.qkv, c->h, D.nqkv, D.d, M, ep, PC_QKV)) != cudaSuccess) return e;
     if (qkv_partial) {
       prof_begin(c, PC_QKV);
-      e = launch_qkv_finish(sp_qkv, c->pos, c->rope, c->q, kinf, vinf, M, D.Hq, D.Hkv, c->st);
+      e = launch_qkv_finish(sp_qkv, w.b_qkv, c->pos, c->rope, c->q, kinf, vinf, M, D.Hq, D.Hkv, c->st);
       prof_end(c);
       if (e != cudaSuccess) return e;
     }
@@ -1002,6 +1012,7 @@ jf_status jf_create(const jf_model_config* model, const jf_runtime_config* rt, j
     w.dn = at<void>(c, O.w_d[l]);
     w.g_attn = at<float>(c, O.g_attn[l]);
     w.g_mlp = at<float>(c, O.g_mlp[l]);
+    w.b_qkv = D.qkv_bias ? at<void>(c, O.b_qkv[l]) : nullptr;
     if (D.bf16) {
       bool ok = make_tmap(&w.tm_qkv, w.qkv, D.d, D.nqkv, kTileN) && make_tmap(&w.tm_o, w.o, D.nq, D.d, kTileN) &&
                 make_tmap(&w.tm_gu, w.gu, D.d, 2 * D.F, kTileN) && make_tmap(&w.tm_dn, w.dn, D.F, D.d, kTileN);
@@ -1112,11 +1123,14 @@ bool tensor_loc(jf_ctx* c, int tid, TensorLoc* t) {
   const long long big = 1ll << 40;
   *t = TensorLoc{nullptr, 0, 0, big, 0, 0, false};
   if (tid == 0) { t->base = (char*)c->w_embed; t->rows = D.V; t->cols = D.d; return true; }
-  if (tid == 1) { t->base = (char*)c->w_lm; t->rows = D.V; t->cols = D.d; return true; }
+  if (tid == 1) {
+    if (D.tie) return false;  // tied: the embedding (tensor 0) is the LM head
+    t->base = (char*)c->w_lm; t->rows = D.V; t->cols = D.d; return true;
+  }
   if (tid == 2) { t->base = (char*)c->g_final; t->rows = 1; t->cols = D.d; t->gain = true; return true; }
   if (tid < 8) return false;
   const int l = (tid - 8) / 16, w = (tid - 8) % 16;
-  if (l >= D.L || w > 8) return false;
+  if (l >= D.L || w > 11 || (w > 8 && !D.qkv_bias)) return false;
   LayerW& L = c->layers[l];
   switch (w) {
     case 0: t->base = (char*)L.g_attn; t->rows = 1; t->cols = D.d; t->gain = true; return true;
@@ -1128,14 +1142,19 @@ bool tensor_loc(jf_ctx* c, int tid, TensorLoc* t) {
     case 6: t->base = (char*)L.gu; t->rows = D.F; t->cols = D.d; t->grp = 1; t->grp_stride = 2; return true;
     case 7: t->base = (char*)L.gu; t->rows = D.F; t->cols = D.d; t->grp = 1; t->grp_stride = 2; t->grp_off = 1; return true;
     case 8: t->base = (char*)L.dn; t->rows = D.d; t->cols = D.F; return true;
+    case 9: t->base = (char*)L.b_qkv; t->rows = 1; t->cols = D.nq; return true;
+    case 10: t->base = (char*)L.b_qkv + (size_t)D.nq * D.es; t->rows = 1; t->cols = D.nkv; return true;
+    case 11: t->base = (char*)L.b_qkv + (size_t)(D.nq + D.nkv) * D.es; t->rows = 1; t->cols = D.nkv; return true;
   }
   return false;
 }
 
 std::vector<int> all_tids(const Dims& D) {
-  std::vector<int> v = {0, 1, 2};
+  std::vector<int> v = {0};
+  if (!D.tie) v.push_back(1);
+  v.push_back(2);
   for (int l = 0; l < D.L; ++l)
-    for (int w = 0; w < 9; ++w) v.push_back(8 + 16 * l + w);
+    for (int w = 0; w < (D.qkv_bias ? 12 : 9); ++w) v.push_back(8 + 16 * l + w);
   return v;
 }
 
@@ -1164,11 +1183,15 @@ cudaError_t copy_tensor(const TensorLoc& t, int es, void* host, cudaMemcpyKind k
   return to_dev ? cudaMemcpyAsync(dt, ht, (size_t)tail * rb, kind, st) : cudaMemcpyAsync(ht, dt, (size_t)tail * rb, kind, st);
 }
 
+// Version 1: the header below without the last two fields (a model with neither QKV biases nor
+// tied embeddings). Version 2 adds them.
 struct FileHeader {
   char magic[4];
   int32_t version, dtype, n_layers, d_model, n_heads, n_kv_heads, head_dim, d_ff, vocab;
   double rms_eps, rope_theta;
+  int32_t qkv_bias, tie_embeddings;
 };
+constexpr size_t kHeaderV1Bytes = offsetof(FileHeader, qkv_bias);
 
 }  // namespace
 
@@ -1230,8 +1253,9 @@ jf_status jf_save_weights(jf_ctx* c, const char* path) {
   if (!c->weights_ready) return fail(c, JF_ESTATE, "weights not initialised");
   FILE* f = std::fopen(path, "wb");
   if (!f) return fail(c, JF_EIO, "cannot open weight file for writing");
-  FileHeader h = {{'J', 'F', 'W', '1'}, 1, c->mc.dtype, c->mc.n_layers, c->mc.d_model, c->mc.n_heads, c->mc.n_kv_heads,
-                  c->mc.head_dim, c->mc.d_ff, c->mc.vocab, c->mc.rms_eps, c->mc.rope_theta};
+  FileHeader h = {{'J', 'F', 'W', '1'}, 2, c->mc.dtype, c->mc.n_layers, c->mc.d_model, c->mc.n_heads,
+                  c->mc.n_kv_heads, c->mc.head_dim, c->mc.d_ff, c->mc.vocab, c->mc.rms_eps, c->mc.rope_theta,
+                  c->mc.qkv_bias, c->mc.tie_embeddings};
   bool ok = std::fwrite(&h, sizeof(h), 1, f) == 1;
   CK(cudaStreamSynchronize(c->st));
   std::vector<uint8_t> buf;
@@ -1255,14 +1279,19 @@ jf_status jf_load_weights(jf_ctx* c, const char* path) {
   if (!c || !path) return JF_EINVAL;
   FILE* f = std::fopen(path, "rb");
   if (!f) return fail(c, JF_EIO, "cannot open weight file");
-  FileHeader h;
-  if (std::fread(&h, sizeof(h), 1, f) != 1 || std::memcmp(h.magic, "JFW1", 4) != 0 || h.version != 1) {
+  FileHeader h = {};
+  bool hdr = std::fread(&h, kHeaderV1Bytes, 1, f) == 1 && std::memcmp(h.magic, "JFW1", 4) == 0 &&
+             (h.version == 1 || h.version == 2);
+  if (hdr && h.version == 2)
+    hdr = std::fread(reinterpret_cast<char*>(&h) + kHeaderV1Bytes, sizeof(h) - kHeaderV1Bytes, 1, f) == 1;
+  if (!hdr) {
     std::fclose(f);
     return fail(c, JF_EIO, "not a JFW1 weight file");
   }
   if (h.dtype != c->mc.dtype || h.n_layers != c->mc.n_layers || h.d_model != c->mc.d_model ||
       h.n_heads != c->mc.n_heads || h.n_kv_heads != c->mc.n_kv_heads || h.head_dim != c->mc.head_dim ||
-      h.d_ff != c->mc.d_ff || h.vocab != c->mc.vocab) {
+      h.d_ff != c->mc.d_ff || h.vocab != c->mc.vocab || h.qkv_bias != c->mc.qkv_bias ||
+      h.tie_embeddings != c->mc.tie_embeddings) {
     std::fclose(f);
     return fail(c, JF_EIO, "weight file has another model shape");
   }

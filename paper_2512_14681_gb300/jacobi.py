@@ -95,7 +95,7 @@ def trajectory_records(buf, n_iters: int, traj_rows: int):
 def model_config(shape: ModelShape) -> J.ModelConfig:
     return J.ModelConfig(shape.n_layers, shape.d_model, shape.n_heads, shape.n_kv_heads, shape.head_dim,
                          shape.d_ff, shape.vocab, shape.rms_eps, shape.rope_theta,
-                         J.JF_BF16 if shape.bf16 else J.JF_F32)
+                         J.JF_BF16 if shape.bf16 else J.JF_F32, int(shape.qkv_bias), int(shape.tie_embeddings))
 
 
 class Context:

@@ -75,6 +75,17 @@ def test_invalid_configs_rejected_on_host(lib):
     bad = _cfg(I.QWEN7B_BF16)
     bad.dtype = 7
     assert lib.jf_arena_bytes(C.byref(bad), C.byref(rc), C.byref(out)) == J.JF_EINVAL
+    for field in ("qkv_bias", "tie_embeddings"):
+        bad = _cfg(I.QWEN7B_BF16)
+        setattr(bad, field, 2)
+        assert lib.jf_arena_bytes(C.byref(bad), C.byref(rc), C.byref(out)) == J.JF_EINVAL, field
+    # a tied LM head needs no arena of its own: exactly one [V, d] matrix less
+    untied, tied = _cfg(I.QWEN7B_BF16), _cfg(I.QWEN7B_BF16)
+    untied.tie_embeddings, tied.tie_embeddings = 0, 1
+    a_u, a_t = C.c_size_t(), C.c_size_t()
+    assert lib.jf_arena_bytes(C.byref(untied), C.byref(rc), C.byref(a_u)) == J.JF_OK
+    assert lib.jf_arena_bytes(C.byref(tied), C.byref(rc), C.byref(a_t)) == J.JF_OK
+    assert 0 <= a_u.value - a_t.value - 152064 * 3584 * 2 < 4096
     rc_bad = J.RuntimeConfig(0, 2048, 64, 0, None, 0, None)
     assert lib.jf_arena_bytes(C.byref(_cfg(I.QWEN7B_BF16)), C.byref(rc_bad), C.byref(out)) == J.JF_EINVAL
     rc_bad = J.RuntimeConfig(1, 2048, 64, 65, None, 0, None)

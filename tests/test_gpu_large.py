@@ -26,7 +26,9 @@ def _round(shape, v):
 
 def _sampled_weights(ctx, shape, n=64):
     rng = np.random.default_rng(5)
-    tids = [0, 1] + [8 + 16 * l + w for l in (0, shape.n_layers - 1) for w in (1, 2, 3, 4, 6, 7, 8)]
+    head = [0] if shape.tie_embeddings else [0, 1]  # a tied model has no separate LM head
+    per = (1, 2, 3, 4, 6, 7, 8) + ((9, 10, 11) if shape.qkv_bias else ())
+    tids = head + [8 + 16 * l + w for l in (0, shape.n_layers - 1) for w in per]
     bad = 0
     for tid in tids:
         rows, cols = _shape_of(shape, tid)
@@ -43,7 +45,7 @@ def _shape_of(shape, tid):
         return shape.vocab, d
     w = (tid - 8) % 16
     return {1: (qd, d), 2: (kvd, d), 3: (kvd, d), 4: (d, qd), 6: (shape.d_ff, d), 7: (shape.d_ff, d),
-            8: (d, shape.d_ff)}[w]
+            8: (d, shape.d_ff), 9: (1, qd), 10: (1, kvd), 11: (1, kvd)}[w]
 
 
 def _expected_inject_counts(truth, P0, n, p, seed, vocab, max_new):

@@ -1,7 +1,8 @@
 """Forward pass of libjf vs the oracle, through the C ABI (tiny fp32 and small bf16 decoders).
 
 * weights: both sides draw the same counter-based N(0, 0.02) stream; the device copy must equal
-  the oracle's values element for element;
+  the oracle's values element for element (also the Q/K/V biases, for the variants with QKV biases
+  and tied embeddings);
 * logits and final hidden state of one causal forward (Eq. 3) over the cache + in-flight rows:
   max-abs 1e-4 (fp32 model) / 3e-2 (bf16 model);
 * the KV commit (cache trim of Algorithm 1) leaves exactly the cache a prefill of the committed
@@ -17,7 +18,15 @@ from tests.parity import LOGIT_TOL, need_gpu
 
 pytestmark = pytest.mark.gpu
 
-SHAPES = [I.TINY_F32, I.SMALL_BF16]
+SHAPES = [I.TINY_F32, I.SMALL_BF16, I.TINY_F32_BT, I.SMALL_BF16_BT]
+
+
+def _tids(shape, layers):
+    """Tensor ids of the shape (include/jf.h): no LM head when tied, three biases a layer with
+    QKV biases."""
+    head = [0, 2] if shape.tie_embeddings else [0, 1, 2]
+    per = 12 if shape.qkv_bias else 9
+    return head + [8 + 16 * l + w for l in layers for w in range(per)]
 
 
 @pytest.fixture(scope="module", params=SHAPES, ids=lambda s: s.name)
@@ -35,7 +44,7 @@ def pair(request):
 
 def test_weights_equal_oracle(pair):
     shape, ctx, model = pair
-    tids = [0, 1, 2] + [8 + 16 * l + w for l in range(shape.n_layers) for w in range(9)]
+    tids = _tids(shape, range(shape.n_layers))
     for tid in tids:
         ref = model.get_tensor(tid)
         got = ctx.get_weights(tid, 0, ref.size).astype(np.float64)
@@ -178,7 +187,7 @@ def test_weight_file_roundtrip_and_refused_files(pair, tmp_path):
     from paper_2512_14681_gb300 import _lib as J
 
     shape, ctx, model = pair
-    tids = [0, 1, 2] + [8 + w for w in range(9)]  # every tensor kind of layer 0
+    tids = _tids(shape, [0])  # every tensor kind of layer 0
 
     def snap():
         out = {}

@@ -1,6 +1,7 @@
 """Strength of the oracle's transformer pins (no GPU): each plausible mistake below is planted into a
-copy of oracle/jf_oracle.c, compiled on the CPU, and the pins of tests/test_oracle_pins.py must
-fail on it. A mistake that no pin notices would mean a hole in the oracle's checks."""
+copy of oracle/jf_oracle.c, compiled on the CPU, and the pins of tests/test_oracle_pins.py and
+tests/test_oracle_bias_tied.py must fail on it. A mistake that no pin notices would mean a hole in
+the oracle's checks. A mistake is one (anchor, replacement) pair, or a list of them."""
 import inspect
 import os
 import shutil
@@ -62,23 +63,38 @@ PLANTED = {
                            "    }\n    free(gt);",
                            "for (int j = 0; j < d; j++) h[(long)i * d + j] = RB(x[(long)i * d + j]);\n"
                            "    }\n    free(gt);"),
+    "query bias dropped": ("for (int j = 0; j < qd; j++) q[(long)i * qd + j] += orc_w(bq, j);", "(void)bq;"),
+    "key bias dropped": ("kk[(long)i * kvd + j] += orc_w(bk, j);", "(void)bk;"),
+    "value bias dropped": ("vv[(long)i * kvd + j] += orc_w(bv, j);", "(void)bv;"),
+    "query and key biases added after the rotary embedding": [
+        ("if (cf->qkv_bias) {\n            /* per-feature biases", "if (0) {\n            /* per-feature biases"),
+        ("            for (int j = 0; j < qd; j++) q[(long)i * qd + j] = RB(q[(long)i * qd + j]);",
+         "            if (cf->qkv_bias) {\n"
+         "                for (int j = 0; j < qd; j++) q[(long)i * qd + j] += orc_w(orc_layer_t(m, l, L_BQ), j);\n"
+         "                for (int j = 0; j < kvd; j++) kk[(long)i * kvd + j] += orc_w(orc_layer_t(m, l, L_BK), j);\n"
+         "                for (int j = 0; j < kvd; j++) vv[(long)i * kvd + j] += orc_w(orc_layer_t(m, l, L_BV), j);\n"
+         "            }\n"
+         "            for (int j = 0; j < qd; j++) q[(long)i * qd + j] = RB(q[(long)i * qd + j]);")],
 }
 
 
 def _pins():
+    import tests.test_oracle_bias_tied as B
     import tests.test_oracle_pins as T
 
-    return [(n, f) for n, f in inspect.getmembers(T, inspect.isfunction)
+    return [(f"{mod.__name__}.{n}", f) for mod in (T, B) for n, f in inspect.getmembers(mod, inspect.isfunction)
             if n.startswith("test_") and not inspect.signature(f).parameters]
 
 
 @pytest.mark.parametrize("name", sorted(PLANTED))
 def test_planted_mistake_fails_a_pin(name, tmp_path, monkeypatch):
-    a, b = PLANTED[name]
+    edits = PLANTED[name]
     src = open(OB.SRC).read()
-    assert src.count(a) == 1, "anchor of the planted mistake not found once"
+    for a, b in ([edits] if isinstance(edits, tuple) else edits):
+        assert src.count(a) == 1, "anchor of the planted mistake not found once"
+        src = src.replace(a, b)
     c_path = tmp_path / "jf_oracle_planted.c"
-    c_path.write_text(src.replace(a, b))
+    c_path.write_text(src)
     so = str(tmp_path / "libjforacle_planted.so")
     subprocess.run(["gcc", "-O2", "-std=c11", "-fopenmp", "-fPIC", "-shared", "-ffp-contract=off", "-o", so,
                     str(c_path), "-lm"], check=True, capture_output=True)

@@ -1,7 +1,8 @@
 """Byte counts behind the bench's roofline, pinned to the model shapes' closed forms.
 
 One Jacobi iteration streams every weight matrix once (q, k, v, o, gate, up, down per layer, the
-LM head, the fp32 norm gains) and reads the committed K/V of every layer; the iteration's roofline
+Q/K/V biases, the LM head (the embedding matrix when tied), the fp32 norm gains) and reads the
+committed K/V of every layer; the iteration's roofline
 is those bytes over the HBM bandwidth. The figures below are the Qwen2.5 shapes' own sizes (7B:
 3584 wide, 28 query / 4 KV heads of 128, SwiGLU 18944, vocabulary 152064, 28 layers; 1.5B: 1536,
 12 / 2, 8960, 151936, 28).
@@ -15,8 +16,9 @@ def test_7b_layer_parameters_and_iteration_bytes():
     attn = 3584 * (28 + 2 * 4) * 128 + 28 * 128 * 3584        # q, k, v, o
     mlp = 3 * 3584 * 18944                                    # gate, up, down
     assert attn + mlp == 233_046_016                          # 233.05 M parameters a layer
+    bias = (28 + 2 * 4) * 128                                 # q, k, v biases
     lm = 152064 * 3584
-    assert s.weight_bytes() == 2 * (28 * (attn + mlp) + lm) + 4 * 3584 * 57
+    assert s.weight_bytes() == 2 * (28 * (attn + mlp + bias) + lm) + 4 * 3584 * 57
     assert abs(s.weight_bytes() / 1e9 - 14.141) < 0.001
 
 
@@ -27,8 +29,8 @@ def test_kv_bytes_per_token():
 
 def test_15b_iteration_bytes():
     s = I.QWEN15B_BF16
-    per_layer = 1536 * (12 + 4) * 128 + 12 * 128 * 1536 + 3 * 1536 * 8960
-    assert s.weight_bytes() == 2 * (28 * per_layer + 151936 * 1536) + 4 * 1536 * 57
+    per_layer = 1536 * (12 + 4) * 128 + 12 * 128 * 1536 + 3 * 1536 * 8960 + (12 + 4) * 128
+    assert s.weight_bytes() == 2 * (28 * per_layer + 151936 * 1536) + 4 * 1536 * 57  # tied: the head is read once
     assert abs(s.weight_bytes() / 1e9 - 3.087) < 0.001
 
 

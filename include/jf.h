@@ -68,12 +68,20 @@ typedef struct {
 /* Capacity. max_rows: in-flight rows per forward (K*n + candidates, or a prefill chunk);
  * max_ctx: positions per sequence (KV pages of 16 tokens are reserved for it; at most 130944
  *   for JF_BF16 models, whose attention stages a sequence's page ids in shared memory);
- * logits_rows: rows jf_forward_logits() may return (0 = that call is unavailable). */
+ * logits_rows: rows jf_forward_logits() may return (0 = that call is unavailable);
+ * page_size: tokens per KV page, 0 or 16 (the only size the kernels support; others are
+ *   JF_EUNSUPPORTED);
+ * max_segments: attention chains one forward may hold, i.e. over all sequences the real-active
+ *   draft with its pseudo-active blocks (one chain) plus every verified candidate (one chain each);
+ *   0 = min(256, 5 * max_seqs + 1), at most 256. It sizes the attention's lane-state scratch;
+ *   calls that would need more return JF_ECAPACITY. */
 typedef struct {
   int max_seqs, max_ctx, max_rows, logits_rows;
   void* device_arena;
   size_t arena_bytes;
   void* cuda_stream;
+  int page_size;
+  int max_segments;
 } jf_runtime_config;
 
 typedef struct jf_ctx jf_ctx;

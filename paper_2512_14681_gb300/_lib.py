@@ -46,7 +46,8 @@ class ModelConfig(C.Structure):
 
 class RuntimeConfig(C.Structure):
     _fields_ = [("max_seqs", C.c_int), ("max_ctx", C.c_int), ("max_rows", C.c_int), ("logits_rows", C.c_int),
-                ("device_arena", C.c_void_p), ("arena_bytes", C.c_size_t), ("cuda_stream", C.c_void_p)]
+                ("device_arena", C.c_void_p), ("arena_bytes", C.c_size_t), ("cuda_stream", C.c_void_p),
+                ("page_size", C.c_int), ("max_segments", C.c_int)]
 
 
 class Block(C.Structure):

@@ -157,7 +157,15 @@ jf_status make_dims(const jf_model_config* m, const jf_runtime_config* rt, Dims*
   D->qkv_bias = m->qkv_bias != 0; D->tie = m->tie_embeddings != 0;
   D->R = rt->max_rows; D->S = rt->max_seqs; D->max_ctx = rt->max_ctx;
   D->pps = cdiv(rt->max_ctx, kPage); D->n_pages = D->S * D->pps; D->logits_rows = rt->logits_rows;
-  D->max_chains = std::min(kMaxChains, D->S * 5 + 1);
+  if (rt->page_size != 0 && rt->page_size != kPage) {
+    *why = "page_size must be 16 (or 0 for the default)";
+    return JF_EUNSUPPORTED;
+  }
+  if (rt->max_segments < 0 || rt->max_segments > kMaxChains) {
+    *why = "max_segments out of range (0 = default, at most 256)";
+    return JF_EINVAL;
+  }
+  D->max_chains = rt->max_segments > 0 ? rt->max_segments : std::min(kMaxChains, D->S * 5 + 1);
   if (D->bf16) {
     D->max_units = D->Hkv * (cdiv((long long)D->R * D->G, kAttnQRows) + D->max_chains);
   } else {
@@ -766,6 +774,8 @@ jf_status generate_impl(jf_ctx* c, int n_seqs, const int32_t* const* h_prompts, 
   const int G = p.ngram_len > 0 ? p.ngram_len : p.block_size;
   const int C = p.pool_size > 0 ? p.cand_per_iter : 0;
   const int rows_per_seq = p.n_blocks * p.block_size + C * G;  // at the largest block size
+  if ((long long)n_seqs * (1 + C) > D.max_chains)
+    return fail(c, JF_ECAPACITY, "more attention chains (sequences x (1 + candidates)) than max_segments");
   // per-sequence block sizes (serving several requests at once) and late joins (chunked prefill
   // inside the decode iterations)
   const int chunk = p.prefill_chunk > 0 ? p.prefill_chunk : std::min(64, D.R);

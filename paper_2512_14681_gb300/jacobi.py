@@ -102,7 +102,7 @@ class Context:
     """A libjf context on the current CUDA device."""
 
     def __init__(self, shape: ModelShape, max_seqs: int = 1, max_ctx: int = 2048, max_rows: int = 64,
-                 logits_rows: int = 0, stream=None):
+                 logits_rows: int = 0, stream=None, max_segments: int = 0):
         import torch
 
         self.lib = J.load()
@@ -110,7 +110,8 @@ class Context:
         self.mc = model_config(shape)
         self.torch = torch
         self.stream = stream if stream is not None else torch.cuda.Stream()
-        rc = J.RuntimeConfig(max_seqs, max_ctx, max_rows, logits_rows, None, 0, self.stream.cuda_stream)
+        rc = J.RuntimeConfig(max_seqs, max_ctx, max_rows, logits_rows, None, 0, self.stream.cuda_stream, 16,
+                             max_segments)
         nbytes = C.c_size_t()
         _check(self.lib, None, self.lib.jf_arena_bytes(C.byref(self.mc), C.byref(rc), C.byref(nbytes)))
         self.arena = torch.empty(nbytes.value, dtype=torch.uint8, device="cuda")

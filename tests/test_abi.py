@@ -88,6 +88,19 @@ def test_invalid_configs_rejected_on_host(lib):
     assert 0 <= a_u.value - a_t.value - 152064 * 3584 * 2 < 4096
     rc_bad = J.RuntimeConfig(0, 2048, 64, 0, None, 0, None)
     assert lib.jf_arena_bytes(C.byref(_cfg(I.QWEN7B_BF16)), C.byref(rc_bad), C.byref(out)) == J.JF_EINVAL
+    for page_size, want in ((16, J.JF_OK), (0, J.JF_OK), (32, J.JF_EUNSUPPORTED), (8, J.JF_EUNSUPPORTED)):
+        r = J.RuntimeConfig(1, 2048, 64, 0, None, 0, None, page_size)
+        assert lib.jf_arena_bytes(C.byref(_cfg(I.QWEN7B_BF16)), C.byref(r), C.byref(out)) == want, page_size
+    for max_segments, want in ((0, J.JF_OK), (1, J.JF_OK), (256, J.JF_OK), (257, J.JF_EINVAL), (-1, J.JF_EINVAL)):
+        r = J.RuntimeConfig(1, 2048, 64, 0, None, 0, None, 16, max_segments)
+        assert lib.jf_arena_bytes(C.byref(_cfg(I.QWEN7B_BF16)), C.byref(r), C.byref(out)) == want, max_segments
+    # max_segments sizes the attention's lane-state scratch: more segments, a larger arena
+    small, large = C.c_size_t(), C.c_size_t()
+    lib.jf_arena_bytes(C.byref(_cfg(I.QWEN7B_BF16)), C.byref(J.RuntimeConfig(1, 2048, 64, 0, None, 0, None, 16, 2)),
+                       C.byref(small))
+    lib.jf_arena_bytes(C.byref(_cfg(I.QWEN7B_BF16)), C.byref(J.RuntimeConfig(1, 2048, 64, 0, None, 0, None, 16, 64)),
+                       C.byref(large))
+    assert large.value > small.value
     rc_bad = J.RuntimeConfig(1, 2048, 64, 65, None, 0, None)
     assert lib.jf_arena_bytes(C.byref(_cfg(I.QWEN7B_BF16)), C.byref(rc_bad), C.byref(out)) == J.JF_EINVAL
     # a context needs an arena

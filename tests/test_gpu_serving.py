@@ -127,3 +127,32 @@ def test_serving_parameters_are_checked(setup):
         with pytest.raises(J.JfError) as ei:
             ctx.generate(prompts, g)
         assert ei.value.status == J.JF_EINVAL
+
+
+def test_max_segments_bounds_the_chains():
+    """jf_runtime_config.max_segments: a context sized for 3 attention chains decodes one sequence
+    with two recycled candidates a forward (3 chains) exactly as a default-sized one does, and
+    refuses two such sequences (6 chains) with JF_ECAPACITY before any launch."""
+    need_gpu()
+    from paper_2512_14681_gb300 import _lib as J
+    from paper_2512_14681_gb300.jacobi import Context, Gen
+
+    shape = I.SMALL_BF16
+    gen = Gen(block_size=8, pool_size=16, cand_per_iter=2, max_new=32)
+    prompts = [I.prompt_tokens(shape.vocab, 24, seed=90 + i) for i in range(2)]
+    ref = Context(shape, max_seqs=2, max_ctx=256, max_rows=64)
+    small = Context(shape, max_seqs=2, max_ctx=256, max_rows=64, max_segments=3)
+    try:
+        for c in (ref, small):
+            c.init_random_weights(I.WEIGHT_SEED, I.WEIGHT_STD)
+        a = ref.generate([prompts[0]], gen)
+        b = small.generate([prompts[0]], gen)
+        assert np.array_equal(a.tokens, b.tokens) and np.array_equal(a.counts, b.counts)
+        with pytest.raises(J.JfError) as ei:
+            small.generate(prompts, gen)
+        assert ei.value.status == J.JF_ECAPACITY
+        c2 = small.generate([prompts[0]], gen)  # the refused call changed nothing
+        assert np.array_equal(c2.tokens, a.tokens)
+    finally:
+        ref.close()
+        small.close()

@@ -151,10 +151,18 @@ __global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(float* __restrict__ x,
   __shared__ float red[NORM_THREADS / 32];
   JF_TL_ENTRY();
   pdl_launch_dependents();  // the next projection may launch now and prefetch its weights
+  const int nv = d >> 2;
+  // the gains are weights (written before this forward began): fetched before the dependency wait
+  const float4* g4 = reinterpret_cast<const float4*>(gain);
+  float4 gv[NORM_VEC];
+#pragma unroll
+  for (int j = 0; j < NORM_VEC; ++j) {
+    const int i = threadIdx.x + j * NORM_THREADS;
+    gv[j] = (i < nv) ? g4[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
   pdl_wait();
   JF_TL_WAITED();
   const int r = row0 + blockIdx.x;
-  const int nv = d >> 2;
   float4* xr = reinterpret_cast<float4*>(x + (size_t)r * d);
   float4 v[NORM_VEC];
 #pragma unroll
@@ -205,13 +213,12 @@ __global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(float* __restrict__ x,
 #pragma unroll
   for (int w = 0; w < NORM_THREADS / 32; ++w) tot += red[w];
   const float rs = 1.0f / sqrtf(tot / (float)d + eps);
-  const float4* g4 = reinterpret_cast<const float4*>(gain);
   T* yr = y + (size_t)blockIdx.x * d;
 #pragma unroll
   for (int j = 0; j < NORM_VEC; ++j) {
     const int i = threadIdx.x + j * NORM_THREADS;
     if (i < nv) {
-      const float4 g = g4[i];
+      const float4 g = gv[j];
       store4(yr + 4 * i, make_float4(v[j].x * rs * g.x, v[j].y * rs * g.y, v[j].z * rs * g.z, v[j].w * rs * g.w));
     }
   }
@@ -231,13 +238,27 @@ __global__ void __launch_bounds__(128) k_qkv_finish(SplitPartials sp, const bf16
                                                      int Hkv) {
   JF_TL_ENTRY();
   pdl_launch_dependents();
-  pdl_wait();
-  JF_TL_WAITED();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int slots = Hq + 2 * Hkv;
   const int job = blockIdx.x * 4 + warp;
   if (job >= M * slots) return;
   const int m = job / slots, hs = job % slots;
+  const bool rot = hs < Hq + Hkv;
+  // before the dependency wait: the bias (a weight), the row's position (written before this
+  // forward's kernels: by a host copy, or by the state machine after the previous forward) and its
+  // rotary coefficients (a table built at context creation)
+  uint2 bw = make_uint2(0u, 0u);
+  if (bias != nullptr) bw = *reinterpret_cast<const uint2*>(bias + (size_t)hs * 128 + lane * 4);
+  float2 c0 = make_float2(1.f, 0.f), c1 = c0, c2 = c0, c3 = c0;
+  if (rot) {
+    const float2* cs = rope + (size_t)pos[m] * 64 + ((lane * 4) & 63);
+    c0 = cs[0];
+    c1 = cs[1];
+    c2 = cs[2];
+    c3 = cs[3];
+  }
+  pdl_wait();
+  JF_TL_WAITED();
   const float* base = sp.ws + ((size_t)(hs * sp.m_tiles + m / sp.bn) * sp.k_splits * sp.bn + (size_t)(m % sp.bn)) * 128 +
                       lane * 4;
   // all partials in flight at once, then added in split order
@@ -256,20 +277,15 @@ __global__ void __launch_bounds__(128) k_qkv_finish(SplitPartials sp, const bf16
     }
   }
   if (bias != nullptr) {  // per-feature bias (bf16 values), after the projection, before RoPE
-    const uint2 w = *reinterpret_cast<const uint2*>(bias + (size_t)hs * 128 + lane * 4);
-    a.x += __uint_as_float(w.x << 16);
-    a.y += __uint_as_float(w.x & 0xffff0000u);
-    a.z += __uint_as_float(w.y << 16);
-    a.w += __uint_as_float(w.y & 0xffff0000u);
+    a.x += __uint_as_float(bw.x << 16);
+    a.y += __uint_as_float(bw.x & 0xffff0000u);
+    a.z += __uint_as_float(bw.y << 16);
+    a.w += __uint_as_float(bw.y & 0xffff0000u);
   }
   bf16* dst;
-  if (hs < Hq + Hkv) {
-    const int p = pos[m];
+  if (rot) {
     const float4 b = make_float4(__shfl_xor_sync(0xffffffffu, a.x, 16), __shfl_xor_sync(0xffffffffu, a.y, 16),
                                  __shfl_xor_sync(0xffffffffu, a.z, 16), __shfl_xor_sync(0xffffffffu, a.w, 16));
-    const int i0 = (lane * 4) & 63;
-    const float2* cs = rope + (size_t)p * 64 + i0;
-    const float2 c0 = cs[0], c1 = cs[1], c2 = cs[2], c3 = cs[3];
     if (lane < 16) {
       a = make_float4(a.x * c0.x - b.x * c0.y, a.y * c1.x - b.y * c1.y, a.z * c2.x - b.z * c2.y, a.w * c3.x - b.w * c3.y);
     } else {

@@ -76,9 +76,34 @@ __global__ void k_embed(const T* __restrict__ E, const int* __restrict__ tok, fl
     if (threadIdx.x == 0) jf_set_error(err, JF_DERR_BOUNDS);
     t = 0;
   }
-  const T* src = E + (size_t)t * d;
-  float* dst = x + (size_t)r * d;
-  for (int i = threadIdx.x; i < d; i += blockDim.x) dst[i] = act_to_f32(src[i]);
+  // 16-byte vectors (d is a multiple of 64, so every row starts 128-byte aligned); up to four
+  // vectors a thread are loaded before the first store, so a row costs one round trip to memory
+  constexpr int VE = 16 / sizeof(T);  // elements per vector
+  const uint4* src = reinterpret_cast<const uint4*>(E + (size_t)t * d);
+  float4* dst = reinterpret_cast<float4*>(x + (size_t)r * d);
+  const int nv = d / VE;
+  for (int base = 0; base < nv; base += 4 * (int)blockDim.x) {
+    uint4 w[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int i = base + k * (int)blockDim.x + (int)threadIdx.x;
+      w[k] = (i < nv) ? src[i] : make_uint4(0u, 0u, 0u, 0u);
+    }
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int i = base + k * (int)blockDim.x + (int)threadIdx.x;
+      if (i >= nv) continue;
+      if constexpr (VE == 8) {  // bf16: 8 values -> two float4
+        dst[2 * i] = make_float4(__uint_as_float(w[k].x << 16), __uint_as_float(w[k].x & 0xffff0000u),
+                                 __uint_as_float(w[k].y << 16), __uint_as_float(w[k].y & 0xffff0000u));
+        dst[2 * i + 1] = make_float4(__uint_as_float(w[k].z << 16), __uint_as_float(w[k].z & 0xffff0000u),
+                                     __uint_as_float(w[k].w << 16), __uint_as_float(w[k].w & 0xffff0000u));
+      } else {  // fp32: 4 values
+        dst[i] = make_float4(__uint_as_float(w[k].x), __uint_as_float(w[k].y), __uint_as_float(w[k].z),
+                             __uint_as_float(w[k].w));
+      }
+    }
+  }
   JF_TL_EXIT(TL_EMBED);
 }
 

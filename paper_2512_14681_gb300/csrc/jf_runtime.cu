@@ -12,6 +12,7 @@
 
 #include "../../include/jf.h"
 #include "../../include/jf_ops.h"
+#include "jf_attn_form.h"
 #include "jf_decode.h"
 #include "jf_internal.h"
 
@@ -546,15 +547,10 @@ cudaError_t enqueue_forward(jf_ctx* c, int M, LmMode lm) {
     if (D.bf16) {
       // units of this forward are bounded by its rows: every chain adds at most one partial tile
       const int units_bound = std::min(D.max_units, D.Hkv * (cdiv((long long)M * D.G, kAttnQRows) + c->chains_bound));
-      // The clustered form folds in parallel but holds at most attn_max_clusters units at once
-      // (15 on a GB300: 120 of 152 SMs); the unclustered form uses every SM and folds on one CTA
-      // per unit. Take the unclustered form only when it needs fewer waves of units, for the unit
-      // count of the rows spread evenly over the chains (exact for equal chains).
-      const int cb = std::max(1, c->chains_bound);
-      const int units_est = std::min(units_bound, D.Hkv * cb * (int)cdiv((long long)cdiv(M, cb) * D.G, kAttnQRows));
-      const int waves_cl = cdiv(units_est, std::max(1, c->attn_max_clusters));
-      const int waves_un = cdiv((long long)units_est * kAttnLanes, c->num_sms);
-      e = launch_attn_tc(a, units_bound, waves_cl <= waves_un, c->st);
+      // clustered unless the unclustered form needs fewer waves of units (jf_attn_form.h)
+      const int units_est = attn_units_estimate(M, c->chains_bound, units_bound, D.Hkv, D.G, kAttnQRows);
+      e = launch_attn_tc(a, units_bound, attn_use_clusters(units_est, kAttnLanes, c->attn_max_clusters, c->num_sms),
+                         c->st);
       prof_end(c);
     } else {
       e = launch_attn_f32(a, M, c->st);
